@@ -1,0 +1,199 @@
+"""fp64 CPU oracle of EpiKV's eviction path (test infrastructure only).
+
+This module is test infrastructure.  Only ``tests/``, ``__graft_entry__.smoke()``
+and ``bench.py``'s CPU-baseline leg may import it; the product path (the CUDA
+library and its binding) never does, and shares no code with it.
+
+It is a plain, slow, obviously correct restatement of the paper's definitions
+in float64 with numpy: no blocking, fusion or reordering beyond what each
+definition states.  Each function names the passage it follows.
+
+Readings of points the paper leaves open (labels match the design notes):
+
+R1  band combination: per-layer z-scores averaged within each band, Band A
+    mean minus Band B mean; the singleton bands {10}, {21} give z10 - z21.
+R2  z window: the last min(w, t) values g(t') with 1 <= t' <= t (causal,
+    includes t; position 0 has no predecessor so no g); z(0) := 0.
+R3  standard deviation is the population one (ddof 0); one value gives 0.
+R4  eps = 1e-6 for both the z-score and the Lag-KV normalisation.
+R5  the z numerator is the raw g_l(t) (Eq. 3), not the rolling mean.
+R6  scores are computed once when a token is generated and then frozen.
+R7  budget K counts every kept token: prefill + recency window + the top
+    candidates; recency R = min(cap, floor(K / 4)) with cap = 128.  When
+    prefill + R >= K the window shrinks to max(0, K - P); prefill is never
+    evicted, so if P > K all P prefill tokens are kept.
+R8  ties between equal scores go to the lower slot (earlier position); NaN
+    ranks below every number; -0 equals +0.
+R9  kept tokens stay in ascending position order after compaction.
+R10 Lag-KV: chunks of lag positions at fixed boundaries t = c*lag; token t in
+    chunk c >= 1 is normalised by the per-channel min/max over all positions
+    of chunk c-1; population variance over the head dimension; K and V
+    variances are added; the mean is over (layer, head); u(t) = 0 in chunk 0;
+    the score is the mean of u over the last min(w, t+1) positions <= t.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+Z_EPS = 1e-6
+LAG_EPS = 1e-6
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.2, Eq. 1 -- hidden-state change
+# --------------------------------------------------------------------------
+def hidden_change(h_prev, h):
+    """g = || h(t) - h(t-1) ||_2 for one pair of rows (Eq. 1)."""
+    d = np.asarray(h, dtype=np.float64) - np.asarray(h_prev, dtype=np.float64)
+    return float(np.sqrt(np.sum(d * d)))
+
+
+def hidden_change_trace(rows):
+    """g[t] for t = 1..T-1 of one layer's rows [T, D]; g[0] is NaN (Eq. 1)."""
+    rows = np.asarray(rows, dtype=np.float64)
+    g = np.full(rows.shape[0], np.nan)
+    for t in range(1, rows.shape[0]):
+        g[t] = hidden_change(rows[t - 1], rows[t])
+    return g
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.2, Eq. 3 -- causal rolling z-score
+# --------------------------------------------------------------------------
+def window_zscore(window, eps=Z_EPS):
+    """(g(t) - mu) / (sigma + eps) over a trailing window whose last entry is
+    g(t) (Eq. 3, readings R3-R5)."""
+    w = np.asarray(window, dtype=np.float64)
+    mu = np.mean(w)
+    sigma = np.sqrt(np.mean((w - mu) ** 2))
+    return float((w[-1] - mu) / (sigma + eps))
+
+
+def rolling_zscore(g, w=64, eps=Z_EPS):
+    """z[t] for a trace of g values indexed by position (Eq. 3, reading R2)."""
+    g = np.asarray(g, dtype=np.float64)
+    z = np.zeros(g.shape[0])
+    for t in range(1, g.shape[0]):
+        z[t] = window_zscore(g[max(1, t - w + 1): t + 1], eps)
+    return z
+
+
+def epiphany_score(z_band_a, z_band_b):
+    """s = mean_{l in A} z_l - mean_{l in B} z_l (Eq. 3 combination, Fig. 1,
+    reading R1).  Arguments are sequences of per-layer z arrays."""
+    za = np.mean(np.asarray(z_band_a, dtype=np.float64), axis=0)
+    zb = np.mean(np.asarray(z_band_b, dtype=np.float64), axis=0)
+    return za - zb
+
+
+def bandz_scores(rows_a, rows_b, w=64, eps=Z_EPS):
+    """EpiKV score of every position 0..T-1 of one sequence.
+
+    rows_a / rows_b: lists of [T, D] arrays, one per Band A / Band B layer.
+    """
+    za = [rolling_zscore(hidden_change_trace(r), w, eps) for r in rows_a]
+    zb = [rolling_zscore(hidden_change_trace(r), w, eps) for r in rows_b]
+    return epiphany_score(za, zb)
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.3 -- Lag-KV: lag-normalised key+value variance
+# --------------------------------------------------------------------------
+def lag_token_variance(k_t, v_t, k_prev_chunk, v_prev_chunk, eps=LAG_EPS):
+    """u(t) for one token whose chunk has a predecessor (Sec. 3.3, R10).
+
+    k_t, v_t: [L, H, d] rows of the token; k_prev_chunk, v_prev_chunk:
+    [lag, L, H, d] rows of every position of the previous chunk.
+    """
+    total = None
+    for x, prev in ((k_t, k_prev_chunk), (v_t, v_prev_chunk)):
+        x = np.asarray(x, dtype=np.float64)
+        prev = np.asarray(prev, dtype=np.float64)
+        mn = prev.min(axis=0)
+        mx = prev.max(axis=0)
+        xn = (x - mn) / (mx - mn + eps)                   # per-channel range
+        mu = xn.mean(axis=-1, keepdims=True)
+        var = ((xn - mu) ** 2).mean(axis=-1)              # over head dim, [L, H]
+        total = var if total is None else total + var     # key + value
+    return float(total.mean())                            # over (layer, head)
+
+
+def lag_variance_trace(K, V, lag=16, eps=LAG_EPS):
+    """u[t] for t = 0..T-1 from K, V rows [T, L, H, d]; u = 0 in chunk 0."""
+    T = K.shape[0]
+    u = np.zeros(T)
+    for t in range(lag, T):
+        c = t // lag
+        lo, hi = (c - 1) * lag, c * lag
+        u[t] = lag_token_variance(K[t], V[t], K[lo:hi], V[lo:hi], eps)
+    return u
+
+
+def rolling_mean(u, w=64):
+    """Causal rolling mean over the last min(w, t+1) positions <= t (R10)."""
+    u = np.asarray(u, dtype=np.float64)
+    return np.array([np.mean(u[max(0, t - w + 1): t + 1]) for t in range(u.shape[0])])
+
+
+def lagkv_scores(K, V, lag=16, eps=LAG_EPS, w=64):
+    return rolling_mean(lag_variance_trace(K, V, lag, eps), w)
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.1, Sec. 3.3 and App. D -- top-K retention under the budget
+# --------------------------------------------------------------------------
+def recency_window(K, cap=128):
+    """R = min(128, K/4) (App. D)."""
+    return min(cap, K // 4)
+
+
+def select_kept(scores, K, prefill=0, recency_cap=128):
+    """Ascending kept slot list of one sequence's cache (Sec. 3.1, App. D).
+
+    scores[i] is the frozen score of cache slot i (slots are in position
+    order).  Prefill slots and the trailing recency window are always kept;
+    the remaining budget goes to the highest-scoring other slots (R7, R8).
+    """
+    scores = np.asarray(scores, dtype=np.float64)
+    n = scores.shape[0]
+    if n <= K:
+        return list(range(n))
+    P = min(prefill, n)
+    R = min(recency_window(K, recency_cap), max(0, K - P))
+    M = max(0, K - P - R)
+    candidates = list(range(P, n - R))
+
+    def rank(i):  # NaN last, higher score first, lower slot first
+        s = scores[i]
+        return (1, 0.0, i) if np.isnan(s) else (0, -s, i)
+
+    best = sorted(candidates, key=rank)[:M]          # a full sort, no shortcuts
+    kept = set(range(P)) | set(range(n - R, n)) | set(best)
+    return sorted(kept)
+
+
+# --------------------------------------------------------------------------
+# App. H -- rebuild the cache from the kept entries, in order
+# --------------------------------------------------------------------------
+def compact(rows, kept):
+    """Cache rows after eviction: the kept slots' rows, in slot order."""
+    return np.asarray(rows)[np.asarray(kept, dtype=np.int64)]
+
+
+def simulate_decode(scores, length, chunk, K, trigger, prefill=0, recency_cap=128):
+    """Replay one sequence's decode: append ``chunk`` tokens at a time and
+    evict whenever the cache holds more than ``trigger`` tokens.
+
+    scores: frozen score of every position (R6).  Returns the list of events
+    as (positions before, positions after) and the final position list.
+    """
+    cache = []
+    events = []
+    for start in range(0, length, chunk):
+        cache.extend(range(start, min(length, start + chunk)))
+        if len(cache) > trigger:
+            kept = select_kept([scores[p] for p in cache], K, prefill, recency_cap)
+            after = [cache[i] for i in kept]
+            events.append((list(cache), after))
+            cache = list(after)
+    return events, cache
