@@ -1,0 +1,420 @@
+#!/usr/bin/env python
+"""Throughput of the EpiKV eviction hot path on GB300.
+
+Workload (the 32k-context decode configuration): 32 sequences, 32 layers x 8
+KV heads x 128 dims bf16 K/V in a paged pool of 16-token blocks with shuffled
+block tables, budget K = 8192, Lag-KV scores (lag 16, rolling window 64).
+One step = the steady-state decode chunk of every sequence: 128 new tokens
+per sequence are scored, each cache (8,320 tokens) is cut back to K and every
+layer's K and V are compacted in place -- one epikv_step through the C ABI
+(Lag-KV partial kernel, finalize kernel, select kernel, TMA compaction kernel).
+
+Inputs are resident in HBM before timing: the 8,192-token caches and the new
+tokens of every timed step (pre-generated into fresh pool blocks that each
+step's block table points to, as a paged serving loop appends tokens).  The
+cache and pool (tens of GB) are far larger than L2, so no flush is needed.
+
+`value` = tokens scored per second over the timed steps (all ranks);
+`e2e` = the same through the same call with the new tokens' K/V copied from
+pinned host memory every step and the new cache lengths read back;
+`roofline` = the compaction kernel's algorithmic bytes (2 x moved rows x
+128 KiB) per launch over its CUDA-event duration, against the measured HBM
+copy bandwidth.  `--impl reference` times the fp64 CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "eviction tokens/s (score+z+top-K+compact)"
+UNIT = "tokens/s"
+WORKLOAD = "batch32_32k_lagkv_paged16_K8192_chunk128"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=20)
+    return p.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+def measured_hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def ncu_traffic(kernel):
+    """Per-launch DRAM bytes from the committed ncu summary, or None when the
+    kernel's source changed since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    src = os.path.join(ROOT, "paper_2606_26472_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("compact.cu", "common.cuh"):
+        h.update(open(os.path.join(src, f), "rb").read())
+    for line in open(path):
+        parts = line.split()
+        if len(parts) == 3 and parts[0] == kernel and parts[1] == h.hexdigest()[:16]:
+            return float(parts[2])
+    return None
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during timing."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id   # the device's UUID ("GPU-...") so no other GPU is sampled
+        self.proc = None
+
+    def start(self):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.count(",") >= 8]
+        os.unlink(self.f.name)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" == r[5 + i].strip()})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------- CPU oracle
+def oracle_step_sample(n_seqs, pos0):
+    """Time the fp64 oracle on `n_seqs` sequence-steps of the workload: Lag-KV
+    scores of 128 new tokens, full-sort selection over the 8,320-slot cache and
+    the gather of the kept K/V rows.  Returns (tokens, seconds)."""
+    from oracle import epikv_oracle as O
+    from synth import gen, workloads as W
+
+    wl = W.config(3)
+    m = wl.model
+    tabs = gen.make_tables(m)
+    K, C, lag, w = wl.budgets[0], wl.chunk, wl.lag, wl.lag_window
+    n_slots = K + C
+    shape = (n_slots, m.num_layers, m.num_kv_heads, m.head_dim)
+    cache_k = np.ones(shape, np.uint16)       # gather cost does not depend on the bytes
+    cache_v = np.ones(shape, np.uint16)
+    first = (pos0 - (w - 1)) // lag * lag - lag  # rows the u window and its ranges reach
+    positions = np.arange(first, pos0 + C)
+    elapsed = 0.0
+    tokens = 0
+    for b in range(n_seqs):
+        sp = gen.spike_flags(m, b, pos0 + C)
+        Kr = gen.bf16_bits_to_f64(gen.kv_rows(m, tabs, b, 0, positions, sp))
+        Vr = gen.bf16_bits_to_f64(gen.kv_rows(m, tabs, b, 1, positions, sp))
+        old = np.random.default_rng(b).normal(size=K)   # frozen scores of the cached tokens
+        t0 = time.perf_counter()
+        u = {}
+        for t in range(pos0 - (w - 1), pos0 + C):
+            c = t // lag
+            lo = (c - 1) * lag - first
+            u[t] = O.lag_token_variance(Kr[t - first], Vr[t - first], Kr[lo:lo + lag], Vr[lo:lo + lag])
+        s_new = [np.mean([u[t - k] for k in range(w)]) for t in range(pos0, pos0 + C)]
+        scores = np.concatenate([old, s_new])
+        kept = O.select_kept(scores, K, 0, wl.recency_cap)
+        O.compact(cache_k, kept)
+        O.compact(cache_v, kept)
+        elapsed += time.perf_counter() - t0
+        tokens += C
+    return tokens, elapsed
+
+
+def cpu_baseline(target_s=12.0):
+    n = 1
+    tok, sec = oracle_step_sample(1, 8192 + 128)
+    while sec < target_s and n < 32:
+        more = min(32 - n, max(1, int((target_s - sec) / max(sec / n, 1e-3))))
+        t2, s2 = oracle_step_sample(more, 8192 + 128)
+        tok, sec, n = tok + t2, sec + s2, n + more
+    return {"value": tok / sec, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} of 32 sequences x 1 decode step (128 tokens: fp64 Lag-KV u over 191 positions + "
+                      f"rolling mean, full-sort selection over 8320 slots, gather of the 8192 kept K and V rows "
+                      f"of 32 layers), {sec:.1f} s of single-threaded numpy"}
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    budget_s = 180.0
+    tok, sec = oracle_step_sample(1, 8192 + 128)   # one warm-up sample
+    steps = max(1, min(args.steps, int(budget_s / max(sec, 1e-3))))
+    tot_tok, tot_s = 0, 0.0
+    for i in range(steps):
+        t, s = oracle_step_sample(1, 8192 + 128 * (i + 2))
+        tot_tok += t
+        tot_s += s
+    v = tot_tok / tot_s
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": steps, "warmup": 1, "ms_per_step": 1e3 * tot_s / steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "oracle_step": "one sequence's decode step"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{steps} sequence-steps of the workload, single-threaded numpy fp64"},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- GPU arm
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    from paper_2606_26472_gb300.cache import KVCache
+    from synth import gen, workloads as W
+    from synth.device import DeviceTrace
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+
+    wl = W.config(3)
+    m = wl.model
+    Bn, K, C = wl.n_seq, wl.budgets[0], wl.chunk
+    L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
+    bs = wl.block_size
+    T_cap = K + C
+    mb = T_cap // bs
+    common = K // bs
+    fresh = C // bs
+    n_steps = args.warmup + args.steps
+    e2e_steps = 0 if args.no_e2e else args.e2e_steps
+    n_blocks = Bn * common + n_steps * Bn * fresh + (Bn * fresh if e2e_steps else 0)
+    perm = gen.block_permutation(m.seed ^ rank, Bn * common).reshape(Bn, common)
+
+    def table(fresh_base):
+        bt = np.empty((Bn, mb), np.int32)
+        bt[:, :common] = perm
+        bt[:, common:] = fresh_base + np.arange(Bn * fresh, dtype=np.int32).reshape(Bn, fresh)
+        return torch.from_numpy(bt).to(dev)
+
+    tables = [table(Bn * common + st * Bn * fresh) for st in range(n_steps)]
+    e2e_base = Bn * common + n_steps * Bn * fresh
+    cache = KVCache(E.EPIKV_LAYOUT_PAGED, L, H, d, max_seqs=Bn, max_tokens=T_cap, block_size=bs,
+                    num_blocks=n_blocks, block_table=tables[0].cpu().numpy(), device=dev)
+    dt = DeviceTrace(m, dev)
+    stream = torch.cuda.current_stream()
+
+    cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T_cap, max_new_tokens=C, num_layers=L, num_kv_heads=H,
+                        head_dim=d, lag=wl.lag, lag_window=wl.lag_window, recency_cap=wl.recency_cap,
+                        score_kinds=E.EPIKV_SCORE_LAGKV)
+    ws_bytes = E.epikv_workspace_bytes(cfg)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws_bytes)
+    for b in range(Bn):
+        E.epikv_seq_reset(ctx, b, 0, E.EPIKV_SCORE_LAGKV)
+
+    # the first K tokens of every trace, scored in decode chunks (no eviction yet)
+    for b in range(Bn):
+        dt.kv(b, 0, K, 0, cache.k, cache.v, **cache.synth_kwargs(tables[0]))
+    seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
+    cu_new = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * C).contiguous()
+    view0 = cache.view(tables[0])
+    for _ in range(K // C):
+        E.epikv_score_update(ctx, Bn, seq_ids, cu_new, C, None, view0)
+    # every step's new tokens, appended into fresh blocks before timing
+    for st in range(n_steps):
+        for b in range(Bn):
+            dt.kv(b, K + st * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tables[st]))
+    views = [cache.view(t) for t in tables]
+    budget = torch.full((Bn,), K, dtype=torch.int32, device=dev)
+    trigger = torch.full((Bn,), K + C - 1, dtype=torch.int32, device=dev)
+    n_out = torch.empty(Bn, dtype=torch.int32, device=dev)
+    torch.cuda.synchronize()
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code} during set-up"
+
+    def step(st, view):
+        E.epikv_step(ctx, Bn, seq_ids, cu_new, C, budget, trigger, None, view, n_out)
+
+    for st in range(args.warmup):
+        step(st, views[st])
+    torch.cuda.synchronize()
+    stats0 = E.epikv_get_stats(ctx)
+
+    def new_events():
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        for e in evs:
+            e.record(stream)   # materialise the handles
+        return evs
+
+    phase = [new_events() for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        gpu_id = str(local_rank)
+    clocks = Clocks(gpu_id)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(args.steps):
+        E.epikv_set_phase_events(ctx, phase[i])
+        step(args.warmup + i, views[args.warmup + i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    E.epikv_set_phase_events(ctx, None)
+    ms = t_start.elapsed_time(t_end)
+    stats1 = E.epikv_get_stats(ctx)
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    t_score = sum(p[0].elapsed_time(p[1]) for p in phase)
+    t_select = sum(p[1].elapsed_time(p[2]) for p in phase)
+    t_compact = sum(p[2].elapsed_time(p[3]) for p in phase)
+    rows_moved = stats1["rows_moved"] - stats0["rows_moved"]
+    tokens = stats1["tokens_scored"] - stats0["tokens_scored"]
+    assert tokens == Bn * C * args.steps
+    row_bytes = L * 2 * H * d * 2                       # one token's K and V, all layers
+    compact_bytes = 2 * rows_moved * row_bytes           # read + write
+    score_bytes = tokens * row_bytes + args.steps * Bn * 2 * (L * 2 * 4 * H * d * 2)  # rows + range state r/w
+
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # ---- end to end: new tokens' K/V from pinned host memory, new lengths back
+    e2e = None
+    if e2e_steps:
+        tab = table(e2e_base)
+        view = cache.view(tab)
+        n_payload = min(4, e2e_steps)
+        payload = torch.empty((n_payload, 2, L, Bn * fresh, bs, H, d), dtype=torch.bfloat16, pin_memory=True)
+        pos_base = K + n_steps * C
+        for j in range(n_payload):
+            for b in range(Bn):
+                dt.kv(b, pos_base + j * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tab))
+            payload[j, 0].copy_(cache.k[:, e2e_base:e2e_base + Bn * fresh])
+            payload[j, 1].copy_(cache.v[:, e2e_base:e2e_base + Bn * fresh])
+        lens = torch.empty((e2e_steps, Bn), dtype=torch.int32, pin_memory=True)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(e2e_steps):
+            src = payload[i % n_payload]
+            for kind, pool in ((0, cache.k), (1, cache.v)):
+                for l in range(L):
+                    pool[l, e2e_base:e2e_base + Bn * fresh].copy_(src[kind, l], non_blocking=True)
+            step(None, view)
+            lens[i].copy_(n_out, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = e0.elapsed_time(e1)
+        if world > 1:
+            t = torch.tensor([e_ms], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_ms = float(t.item())
+        assert (lens.numpy() == K).all()
+        e2e = {"value": world * Bn * C * e2e_steps / (e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(payload[0].numel() * 2), "d2h_bytes_per_step": Bn * 4,
+               "steps": e2e_steps}
+        st_, code = E.epikv_get_error(ctx)
+        assert st_ == E.EPIKV_OK, f"device error {code} in e2e"
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    peak, peak_src = measured_hbm_peak()
+    ach = compact_bytes / args.steps / (t_compact / args.steps / 1e3) / 1e9
+    traffic = ncu_traffic("compact_kernel")
+    line = {
+        "metric": METRIC, "value": world * tokens / (ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sequences": Bn, "context": 32768, "budget_K": K, "chunk": C,
+                   "layers": L, "kv_heads": H, "head_dim": d, "kv_dtype": "bf16", "layout": "paged16_shuffled",
+                   "score": "lagkv_lag16_w64", "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
+        "compaction_gbs": ach,
+        "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
+                                "compact": t_compact / args.steps},
+        "step_hbm_gbs": (compact_bytes + score_bytes) / (ms / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
+                     "frac": ach / peak, "peak_source": peak_src,
+                     "traffic": traffic, "algorithmic_bytes_per_launch": compact_bytes / args.steps},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline()
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

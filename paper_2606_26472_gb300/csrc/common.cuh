@@ -1,0 +1,176 @@
+// Device-side helpers shared by the EpiKV kernels: the context's device
+// state, K/V row addressing for both layouts, the sticky error word, and
+// inline-PTX wrappers for 1-D TMA bulk copies and mbarriers (sm_90+ ISA,
+// compiled here for sm_103a only).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "epikv.h"
+
+namespace epikv {
+
+constexpr int kMaxBand = 32;
+
+// Device pointers carved out of the caller's workspace (one context).
+struct DevState {
+  int32_t* n_cache;        // [S] slots in use
+  int32_t* n_seen;         // [S] next position
+  int32_t* prefill;        // [S]
+  int32_t* policy;         // [S] score kind driving selection (1 or 2)
+  int32_t* hp_parity;      // [S] which h_prev buffer holds the last row
+  int32_t* first_changed;  // [S] first slot moved by the last selection
+  uint32_t* ticket;        // [S] last-CTA tickets of the finalize kernel
+  int32_t* err;            // [1] sticky device error word
+  unsigned long long* stats;  // [4] epikv_stats
+  float* score[2];         // [S][T] frozen scores (kind 0 = band-z, 1 = Lag-KV)
+  int32_t* pos;            // [S][T] position of each slot
+  __nv_bfloat16* h_prev;   // [S][2][n_band][D] last hidden row per band layer
+  float* g_ring;           // [S][n_band][G] g by position (mod G)
+  __nv_bfloat16* lag_rng;  // [S][L][2][4][H][d] prev min, prev max, cur min, cur max
+  float* lag_part;         // [S][max_new][2L] per-(layer, K|V) head-summed variances
+  float* u_ring;           // [S][G] u by position (mod G)
+  int32_t* kept;           // [S][T] kept lists of epikv_step
+  int32_t* n_kept;         // [S]
+};
+
+struct Dims {
+  int S, T, max_new, L, H, d, D, nA, nB, G;
+  int z_window, lag, lag_window, recency_cap, kinds;
+  float z_eps, lag_eps;
+};
+
+struct KvDev {
+  char* base[2];           // K, V
+  int layout;
+  int64_t stride_layer, stride_seq, stride_block, stride_token;  // elements
+  const int32_t* block_table;
+  int max_blocks, block_size, num_blocks;
+};
+
+__device__ __forceinline__ void set_error(int32_t* err, int code) {
+  atomicCAS(err, 0, code);
+}
+
+// Element offset of (layer, seq, slot) or -1 if outside the view.
+__device__ __forceinline__ int64_t kv_row_offset(const KvDev& v, int layer, int seq, int slot, int T) {
+  if (slot < 0) return -1;
+  if (v.layout == EPIKV_LAYOUT_CONTIGUOUS) {
+    if (slot >= T) return -1;
+    return (int64_t)layer * v.stride_layer + (int64_t)seq * v.stride_seq + (int64_t)slot * v.stride_token;
+  }
+  int bi = slot / v.block_size;
+  if (bi >= v.max_blocks) return -1;
+  int blk = __ldg(v.block_table + (int64_t)seq * v.max_blocks + bi);
+  if (blk < 0 || blk >= v.num_blocks) return -1;
+  return (int64_t)layer * v.stride_layer + (int64_t)blk * v.stride_block +
+         (int64_t)(slot - bi * v.block_size) * v.stride_token;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ void unpack8(const uint4& q, float* f) {
+  f[0] = bf16_lo(q.x); f[1] = bf16_hi(q.x);
+  f[2] = bf16_lo(q.y); f[3] = bf16_hi(q.y);
+  f[4] = bf16_lo(q.z); f[5] = bf16_hi(q.z);
+  f[6] = bf16_lo(q.w); f[7] = bf16_hi(q.w);
+}
+
+// Streaming 16-byte load that does not allocate in L1.
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+  return r;
+}
+
+// ---------------------------------------------------------------- mbarrier
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;"
+               :: "r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+
+// One probe (the hardware may suspend the thread for up to ~1 us); true when
+// the phase with `parity` has completed.
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, 1000;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Wait at most `limit_ns` of wall time; false if it gave up.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_ns() - t0 > limit_ns) return false;
+  return true;
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ------------------------------------------------------------ TMA bulk copies
+// global -> shared, completion counted in bytes on `bar`.
+__device__ __forceinline__ void tma_load_1d(void* smem_dst, const void* gmem_src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      :: "r"(smem_u32(smem_dst)), "l"(gmem_src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+
+// shared -> global, tracked by this thread's bulk async-groups.
+__device__ __forceinline__ void tma_store_1d(void* gmem_dst, const void* smem_src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+               :: "l"(gmem_dst), "r"(smem_u32(smem_src)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void tma_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+
+// Wait until at most N of this thread's bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void tma_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" :: "n"(N) : "memory");
+}
+
+__device__ __forceinline__ void tma_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// ------------------------------------------------------------ warp helpers
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over aligned groups of `width` lanes (width a power of two <= 32).
+__device__ __forceinline__ float group_sum(float v, int width) {
+  for (int o = width >> 1; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+}  // namespace epikv

@@ -1,0 +1,216 @@
+// In-place, order-preserving K/V compaction to the kept set (App. H).
+//
+// For every sequence that evicted in the last selection and every
+// (layer, K|V, head group) stream: row i <- row kept[i] for i from the first
+// evicted slot to the new cache length.  Rows are moved with 1-D TMA bulk
+// copies global -> shared -> global (cp.async.bulk + mbarrier), no cluster
+// multicast.  A persistent grid of one-warp CTAs walks its streams' batches
+// through a ring of shared-memory stages: while batch k is stored, batches
+// k+1 .. k+S-1 are loading.
+//
+// In-place safety without any inter-CTA wait: streams are disjoint bytes, so
+// one CTA owns each; inside a stream kept[i] >= i and rows are processed in
+// increasing i, so a load (slot kept[i] >= i) never reads a slot that an
+// earlier store has written, and a later store to a slot some earlier batch
+// still had to read is issued only after that batch's loads completed.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace epikv {
+
+constexpr int kStageBytes = 16384;
+constexpr int kStages = 4;
+constexpr int kMaxRowsPerLane = 4;
+constexpr int kMaxRPB = 32 * kMaxRowsPerLane;
+constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s: far beyond any real copy
+constexpr uint64_t kDrainNs = 100000000ull;   // 0.1 s per stage after a timeout
+
+struct Cursor {
+  int u;      // unit index (this CTA strides by gridDim.x)
+  int i;      // next row of the unit
+  int end;    // row past the last of the unit
+  int b, seq, layer, kvk, hg;
+};
+
+__global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev kv,
+                                                     const int32_t* __restrict__ seq_ids, int n_seq,
+                                                     const int32_t* __restrict__ kept, int kept_stride) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  __shared__ __align__(8) uint64_t full[kStages];
+  __shared__ char* dptr[kStages][kMaxRPB];
+  __shared__ int stage_rows[kStages];
+  int* list = reinterpret_cast<int*>(smem + kStages * kStageBytes);
+  const int lane = threadIdx.x;
+
+  // ---- the batch entries that evicted (every CTA builds the same list)
+  int n_ev = 0;
+  for (int base = 0; base < n_seq; base += 32) {
+    const int b = base + lane;
+    bool ev = false;
+    if (b < n_seq) {
+      const int seq = seq_ids[b];
+      ev = seq >= 0 && seq < dm.S && st.first_changed[seq] < st.n_cache[seq];
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, ev);
+    if (ev) list[n_ev + __popc(m & ((1u << lane) - 1u))] = b;
+    n_ev += __popc(m);
+  }
+  __syncwarp();
+  if (n_ev == 0) return;
+
+  // ---- head split: the one (1, 2, 4, ...) whose unit count fills the grid best
+  const int G = gridDim.x;
+  int hs = 1;
+  {
+    double best = -1.0;
+    for (int c = 1; c <= dm.H; c <<= 1) {
+      if (dm.H % c != 0 || (dm.H / c) * dm.d * 2 < 256) break;
+      const long units = (long)n_ev * 2 * dm.L * c;
+      const long rounds = (units + G - 1) / G;
+      const double eff = (double)units / (double)(rounds * G);
+      if (eff > best + 1e-3) { best = eff; hs = c; }
+    }
+  }
+  const int rb = (dm.H / hs) * dm.d * 2;               // bytes per row piece
+  const int64_t piece_elems = (int64_t)(dm.H / hs) * dm.d;
+  const int rpb = min(kStageBytes / rb, kMaxRPB);      // rows per batch
+  const int upe = 2 * dm.L * hs;
+  const int units = n_ev * upe;
+
+  if (lane == 0) {
+    for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  __syncwarp();
+
+  auto load_unit = [&](Cursor& c) {
+    while (c.u < units) {
+      const int e = c.u / upe, rem = c.u % upe;
+      c.layer = rem / (2 * hs);
+      c.kvk = (rem / hs) & 1;
+      c.hg = rem % hs;
+      c.b = list[e];
+      c.seq = seq_ids[c.b];
+      c.i = st.first_changed[c.seq];
+      c.end = st.n_cache[c.seq];
+      if (c.i < c.end) return;
+      c.u += G;
+    }
+  };
+  auto advance = [&](Cursor& c) {
+    c.i += rpb;
+    if (c.i >= c.end) {
+      c.u += G;
+      load_unit(c);
+    }
+  };
+
+  // issue the loads of the batch at cursor c into stage s
+  auto issue = [&](const Cursor& c, int s) {
+    const int nrows = min(rpb, c.end - c.i);
+    char* kvb = kv.base[c.kvk];
+    unsigned char* stage = smem + s * kStageBytes;
+    const int32_t* kl = kept + (size_t)c.b * kept_stride;
+    const char* src[kMaxRowsPerLane];
+    uint32_t total = 0;
+#pragma unroll
+    for (int j = 0; j < kMaxRowsPerLane; ++j) {
+      const int r = lane + 32 * j;
+      src[j] = nullptr;
+      bool ok = false;
+      if (r < nrows) {
+        const int i = c.i + r;
+        const int from = kl[i];
+        const int64_t so = from >= i ? kv_row_offset(kv, c.layer, c.seq, from, dm.T) : -1;
+        const int64_t dof = kv_row_offset(kv, c.layer, c.seq, i, dm.T);
+        ok = so >= 0 && dof >= 0;
+        if (ok) {
+          src[j] = kvb + (so + c.hg * piece_elems) * 2;
+          dptr[s][r] = kvb + (dof + c.hg * piece_elems) * 2;
+        } else {
+          dptr[s][r] = nullptr;
+          set_error(st.err, from < i ? EPIKV_DEV_KEPT : EPIKV_DEV_SLOT);
+        }
+      }
+      total += __popc(__ballot_sync(0xffffffffu, ok)) * (uint32_t)rb;
+    }
+    if (lane == 0) {
+      stage_rows[s] = nrows;
+      mbar_arrive_expect_tx(&full[s], total);
+    }
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < kMaxRowsPerLane; ++j)
+      if (src[j]) tma_load_1d(stage + (lane + 32 * j) * rb, src[j], rb, &full[s]);
+  };
+
+  Cursor ld;
+  ld.u = blockIdx.x;
+  load_unit(ld);
+  int k_issue = 0, k_store = 0;
+  bool timed_out = false;
+  for (int p = 0; p < kStages - 1 && ld.u < units; ++p) {
+    issue(ld, k_issue % kStages);
+    ++k_issue;
+    advance(ld);
+  }
+  while (k_store < k_issue) {
+    const int s = k_store % kStages;
+    if (!mbar_wait_bounded(&full[s], (k_store / kStages) & 1, kWaitNs)) {
+      timed_out = true;
+      break;
+    }
+    __syncwarp();
+    const int nrows = stage_rows[s];
+    unsigned char* stage = smem + s * kStageBytes;
+    for (int r = lane; r < nrows; r += 32)
+      if (dptr[s][r]) tma_store_1d(dptr[s][r], stage + r * rb, rb);
+    tma_commit();
+    ++k_store;
+    if (ld.u < units) {
+      tma_wait_read<1>();  // the stage about to be refilled has been read out
+      __syncwarp();
+      issue(ld, k_issue % kStages);
+      ++k_issue;
+      advance(ld);
+    }
+  }
+  if (timed_out) {
+    if (lane == 0) set_error(st.err, EPIKV_DEV_TIMEOUT);
+    // let the loads still in flight land before the CTA's shared memory goes away
+    for (int k = k_store; k < k_issue; ++k)
+      mbar_wait_bounded(&full[k % kStages], (k / kStages) & 1, kDrainNs);
+  }
+  tma_wait_all();
+}
+
+static int g_ctas_per_sm = 0;
+
+static size_t compact_smem(int n_seq) {
+  return (size_t)kStages * kStageBytes + (size_t)((n_seq + 31) / 32 * 32) * sizeof(int);
+}
+
+cudaError_t compact_prepare(int device, int* ctas_per_sm) {
+  (void)device;
+  cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)compact_smem(4096));
+  if (e != cudaSuccess) return e;
+  int n = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, 32, compact_smem(64));
+  if (e != cudaSuccess) return e;
+  g_ctas_per_sm = n > 0 ? n : 1;
+  if (ctas_per_sm) *ctas_per_sm = g_ctas_per_sm;
+  return cudaSuccess;
+}
+
+cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
+                           const int32_t* kept, int kept_stride, const KvDev& kv, int ctas,
+                           cudaStream_t stream, int* launches) {
+  if (n_seq == 0) return cudaSuccess;
+  compact_kernel<<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  ++*launches;
+  return cudaGetLastError();
+}
+
+}  // namespace epikv

@@ -1,0 +1,439 @@
+// Scoring kernels of the EpiKV hot path.
+//
+//   bandz_g_kernel         g_l(t) = ||h_l(t) - h_l(t-1)||_2 of every new token
+//                          and band layer (Sec. 3.2, Eq. 1), streamed from the
+//                          bf16 rows with 16-byte loads, fp32 accumulation.
+//   lagkv_partial_kernel   Lag-KV (Sec. 3.3): each new token's K or V row of one
+//                          layer, normalised by the previous chunk's per-channel
+//                          range; population variance over the head dimension,
+//                          summed over heads.  Keeps the running chunk ranges.
+//   score_finalize_kernel  causal rolling z-score per band layer and the band
+//                          combination (Eq. 3, Fig. 1); Lag-KV u(t) and its
+//                          rolling mean; writes the frozen score and position of
+//                          every new slot and commits the sequence's counters.
+//
+// Every result is independent of how a trace is split into calls: g values
+// and u values are computed from the same bytes in the same order whether the
+// previous row comes from the call or from the saved state, and the window
+// reductions run over positions in a fixed lane order.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace epikv {
+
+constexpr int kGThreads = 256;
+constexpr int kGUnroll = 4;
+
+struct BandRows {
+  const __nv_bfloat16* p[kMaxBand];
+};
+
+// grid: (token tiles, band layers, batch entries); block: 256 threads.
+template <int VPT>
+__global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm, BandRows rows,
+                                                            int64_t row_stride,
+                                                            const int32_t* __restrict__ seq_ids,
+                                                            const int32_t* __restrict__ cu_new,
+                                                            int max_new, int tok_per_cta) {
+  const int b = blockIdx.z, band = blockIdx.y;
+  const int seq = seq_ids[b];
+  const int r0 = cu_new[b];
+  const int n_new = cu_new[b + 1] - r0;
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int t0 = blockIdx.x * tok_per_cta;
+  if (t0 >= n_new) return;
+  const int t1 = min(t0 + tok_per_cta, n_new);
+  const int p0 = st.n_seen[seq];
+  const int par = st.hp_parity[seq];
+  const int nb = dm.nA + dm.nB;
+  const int VR = dm.D >> 3;  // 16-byte vectors per row
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  const __nv_bfloat16* hp_rd = st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D;
+  __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
+  const __nv_bfloat16* base = rows.p[band];
+  float* ring = st.g_ring + ((size_t)seq * nb + band) * dm.G;
+
+  const __nv_bfloat16* prow = (t0 == 0) ? hp_rd : base + (int64_t)(r0 + t0 - 1) * row_stride;
+  uint4 prev[VPT];
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int v = tid + k * kGThreads;
+    prev[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
+  }
+
+  __shared__ float red[kGUnroll][kGThreads / 32];
+  for (int t = t0; t < t1; t += kGUnroll) {
+    uint4 cur[kGUnroll][VPT];
+#pragma unroll
+    for (int u = 0; u < kGUnroll; ++u) {
+      const __nv_bfloat16* row = base + (int64_t)(r0 + t + u) * row_stride;
+#pragma unroll
+      for (int k = 0; k < VPT; ++k) {
+        const int v = tid + k * kGThreads;
+        cur[u][k] = (t + u < t1 && v < VR) ? ld_stream16(row + v * 8) : make_uint4(0, 0, 0, 0);
+      }
+    }
+    float part[kGUnroll];
+#pragma unroll
+    for (int u = 0; u < kGUnroll; ++u) {
+      float acc = 0.f;
+#pragma unroll
+      for (int k = 0; k < VPT; ++k) {
+        float c[8], p[8];
+        unpack8(cur[u][k], c);
+        unpack8(u == 0 ? prev[k] : cur[u - 1][k], p);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float dlt = c[e] - p[e];
+          acc = fmaf(dlt, dlt, acc);
+        }
+      }
+      part[u] = warp_sum(acc);
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int u = 0; u < kGUnroll; ++u) red[u][warp] = part[u];
+    }
+    // the last valid row of this group is the previous row of the next group
+    const int last = min(kGUnroll, t1 - t) - 1;
+#pragma unroll
+    for (int u = 0; u < kGUnroll; ++u)
+      if (u == last) {
+#pragma unroll
+        for (int k = 0; k < VPT; ++k) prev[k] = cur[u][k];
+      }
+    __syncthreads();
+    if (tid < kGUnroll && t + tid < t1) {
+      float s = 0.f;
+#pragma unroll
+      for (int w = 0; w < kGThreads / 32; ++w) s += red[tid][w];
+      const int pos = p0 + t + tid;
+      if (pos >= 1) ring[pos & (dm.G - 1)] = sqrtf(s);
+    }
+    __syncthreads();
+  }
+  if (t1 == n_new) {
+#pragma unroll
+    for (int k = 0; k < VPT; ++k) {
+      const int v = tid + k * kGThreads;
+      if (v < VR) *reinterpret_cast<uint4*>(hp_wr + v * 8) = prev[k];
+    }
+  }
+}
+
+constexpr int kLagBatch = 16;
+
+// grid: (2L (layer, K|V), batch entries); block: max(32, H*d/8) threads,
+// lanes-per-head LH = d/8 consecutive threads own one head (8 channels each).
+template <int LH>
+__global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
+                                                             const int32_t* __restrict__ seq_ids,
+                                                             const int32_t* __restrict__ cu_new,
+                                                             int max_new) {
+  const int b = blockIdx.y;
+  const int seq = seq_ids[b];
+  const int n_new = cu_new[b + 1] - cu_new[b];
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int layer = blockIdx.x >> 1, kvk = blockIdx.x & 1;
+  const int tid = threadIdx.x;
+  const int h = tid / LH, q = tid % LH;
+  const bool active = h < dm.H;
+  const int hd = dm.H * dm.d;
+  const int nc0 = st.n_cache[seq];
+  const int p0 = st.n_seen[seq];
+  if (nc0 + n_new > dm.T) {
+    if (tid == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+    return;
+  }
+  const int ch = h * dm.d + q * 8;  // first channel of this thread within the token row
+  __nv_bfloat16* rng = st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd;
+
+  float pmn[8], pmx[8], cmn[8], cmx[8], inv[8];
+  if (active) {
+    unpack8(*reinterpret_cast<const uint4*>(rng + 0 * hd + ch), pmn);
+    unpack8(*reinterpret_cast<const uint4*>(rng + 1 * hd + ch), pmx);
+    unpack8(*reinterpret_cast<const uint4*>(rng + 2 * hd + ch), cmn);
+    unpack8(*reinterpret_cast<const uint4*>(rng + 3 * hd + ch), cmx);
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) pmn[e] = pmx[e] = cmn[e] = cmx[e] = 0.f;
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) inv[e] = 1.f / (pmx[e] - pmn[e] + dm.lag_eps);
+
+  const float inv_d = 1.f / (float)dm.d;
+  const char* kvbase = kv.base[kvk];
+  __shared__ float hv[kLagBatch][32];  // per token, per head (the host admits H <= 32)
+  float* part = st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L);
+
+  for (int i0 = 0; i0 < n_new; i0 += kLagBatch) {
+    const int nbt = min(kLagBatch, n_new - i0);
+    uint4 x[kLagBatch];
+#pragma unroll
+    for (int j = 0; j < kLagBatch; ++j) {
+      x[j] = make_uint4(0, 0, 0, 0);
+      if (j < nbt && active) {
+        const int64_t off = kv_row_offset(kv, layer, seq, nc0 + i0 + j, dm.T);
+        if (off >= 0)
+          x[j] = ld_stream16(kvbase + (off + ch) * 2);
+        else
+          set_error(st.err, EPIKV_DEV_SLOT);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kLagBatch; ++j) {
+      if (j < nbt) {
+        const int pos = p0 + i0 + j;
+        const int c = pos / dm.lag;
+        const int r = pos - c * dm.lag;
+        float xf[8];
+        unpack8(x[j], xf);
+        float var = 0.f;
+        if (c >= 1) {  // uniform across the block: every thread sees the same token
+          float xn[8], s = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            xn[e] = (xf[e] - pmn[e]) * inv[e];
+            s += xn[e];
+          }
+          const float mean = group_sum(s, LH) * inv_d;
+          float ss = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float dv = xn[e] - mean;
+            ss = fmaf(dv, dv, ss);
+          }
+          var = group_sum(ss, LH) * inv_d;
+        }
+        if (q == 0 && active) hv[j][h] = var;
+        if (r == 0) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) cmn[e] = cmx[e] = xf[e];
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            cmn[e] = fminf(cmn[e], xf[e]);
+            cmx[e] = fmaxf(cmx[e], xf[e]);
+          }
+        }
+        if (r == dm.lag - 1) {  // chunk complete: it becomes the previous chunk
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            pmn[e] = cmn[e];
+            pmx[e] = cmx[e];
+            inv[e] = 1.f / (pmx[e] - pmn[e] + dm.lag_eps);
+          }
+        }
+      }
+    }
+    __syncthreads();
+    if (tid < nbt) {
+      float s = 0.f;
+      for (int hh = 0; hh < dm.H; ++hh) s += hv[tid][hh];
+      part[(size_t)(i0 + tid) * (2 * dm.L) + blockIdx.x] = s;
+    }
+    __syncthreads();
+  }
+  if (active) {
+    auto pack = [](const float* f) {
+      uint4 q4;
+      q4.x = (__float_as_uint(f[0]) >> 16) | (__float_as_uint(f[1]) & 0xFFFF0000u);
+      q4.y = (__float_as_uint(f[2]) >> 16) | (__float_as_uint(f[3]) & 0xFFFF0000u);
+      q4.z = (__float_as_uint(f[4]) >> 16) | (__float_as_uint(f[5]) & 0xFFFF0000u);
+      q4.w = (__float_as_uint(f[6]) >> 16) | (__float_as_uint(f[7]) & 0xFFFF0000u);
+      return q4;  // exact: every value is a bf16 value held in fp32
+    };
+    *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = pack(pmn);
+    *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = pack(pmx);
+    *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = pack(cmn);
+    *reinterpret_cast<uint4*>(rng + 3 * hd + ch) = pack(cmx);
+  }
+}
+
+constexpr int kFinTile = 32;
+constexpr int kFinThreads = 256;
+constexpr int kMaxWindow = 1024;
+
+// grid: (token tiles of 32, batch entries); block: 256 threads (warp per token).
+template <int WPL>
+__global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st, Dims dm,
+                                                                     const int32_t* __restrict__ seq_ids,
+                                                                     const int32_t* __restrict__ cu_new,
+                                                                     int max_new) {
+  const int b = blockIdx.y;
+  const int seq = seq_ids[b];
+  const int n_new = cu_new[b + 1] - cu_new[b];
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nc0 = st.n_cache[seq];
+  const int p0 = st.n_seen[seq];
+  const bool fits = nc0 + n_new <= dm.T;
+  if (!fits && tid == 0 && blockIdx.x == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+  const int i_lo = blockIdx.x * kFinTile;
+  const int i_hi = min(i_lo + kFinTile, n_new);
+  const int Gm = dm.G - 1;
+  const int nb = dm.nA + dm.nB;
+
+  if (fits && i_lo < i_hi) {
+    for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
+      const int pos = p0 + i;
+      if (lane == 0) st.pos[(size_t)seq * dm.T + nc0 + i] = pos;
+    }
+    if (dm.kinds & EPIKV_SCORE_BANDZ) {
+      for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
+        const int pos = p0 + i;
+        float s = 0.f;
+        if (pos >= 1) {
+          const int n = min(dm.z_window, pos);
+          const float inv_n = 1.f / (float)n;
+          float za = 0.f, zb = 0.f;
+          for (int band = 0; band < nb; ++band) {
+            const float* ring = st.g_ring + ((size_t)seq * nb + band) * dm.G;
+            const float gnew = ring[pos & Gm];
+            float v[WPL], dsum = 0.f;
+#pragma unroll
+            for (int m = 0; m < WPL; ++m) {
+              const int k = lane + 32 * m;  // window offset: position pos - k
+              v[m] = k < n ? ring[(pos - k) & Gm] - gnew : 0.f;
+              dsum += v[m];
+            }
+            const float mean_d = warp_sum(dsum) * inv_n;
+            float dev = 0.f;
+#pragma unroll
+            for (int m = 0; m < WPL; ++m) {
+              const int k = lane + 32 * m;
+              if (k < n) {
+                const float e = v[m] - mean_d;
+                dev = fmaf(e, e, dev);
+              }
+            }
+            const float sigma = sqrtf(warp_sum(dev) * inv_n);
+            const float z = -mean_d / (sigma + dm.z_eps);  // g(t) - mu = -(mean of g - g(t))
+            if (band < dm.nA) za += z; else zb += z;
+          }
+          s = za / (float)dm.nA - zb / (float)dm.nB;
+        }
+        if (lane == 0) st.score[0][(size_t)seq * dm.T + nc0 + i] = s;
+      }
+    }
+    if (dm.kinds & EPIKV_SCORE_LAGKV) {
+      __shared__ float su[kFinTile + kMaxWindow];
+      const int w = dm.lag_window;
+      const int lo = max(0, i_lo - (w - 1));
+      const float* part = st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L);
+      const float inv_lh = 1.f / (float)(dm.L * dm.H);
+      for (int i = lo + tid; i < i_hi; i += kFinThreads) {
+        const int pos = p0 + i;
+        float u = 0.f;
+        if (pos >= dm.lag) {
+          const float* pp = part + (size_t)i * (2 * dm.L);
+          float s = 0.f;
+          for (int q = 0; q < 2 * dm.L; ++q) s += pp[q];
+          u = s * inv_lh;
+        }
+        su[i - lo] = u;
+      }
+      __syncthreads();
+      for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
+        const int pos = p0 + i;
+        const int n = min(w, pos + 1);
+        float acc = 0.f;
+#pragma unroll
+        for (int m = 0; m < WPL; ++m) {
+          const int k = lane + 32 * m;
+          if (k < n) acc += (i - k >= 0) ? su[i - k - lo] : st.u_ring[(size_t)seq * dm.G + ((pos - k) & Gm)];
+        }
+        const float mean = warp_sum(acc) / (float)n;
+        if (lane == 0) st.score[1][(size_t)seq * dm.T + nc0 + i] = mean;
+      }
+      for (int i = i_lo + tid; i < i_hi; i += kFinThreads)
+        st.u_ring[(size_t)seq * dm.G + ((p0 + i) & Gm)] = su[i - lo];
+    }
+  }
+
+  // The last CTA of this sequence commits its counters (no CTA waits).
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const uint32_t done = atomicAdd(&st.ticket[seq], 1u);
+    if (done == gridDim.x - 1) {
+      __threadfence();
+      if (fits) {
+        st.n_cache[seq] = nc0 + n_new;
+        st.n_seen[seq] = p0 + n_new;
+        if ((dm.kinds & EPIKV_SCORE_BANDZ) && n_new > 0) st.hp_parity[seq] ^= 1;
+        atomicAdd(&st.stats[0], (unsigned long long)n_new);
+      }
+      st.ticket[seq] = 0u;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ launchers
+cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
+                                const int32_t* cu_new, int max_new, const epikv_hidden_view* hv,
+                                const KvDev* kv, int num_sms, cudaStream_t stream, int* launches) {
+  if (n_seq == 0 || max_new == 0) return cudaSuccess;
+  const int nb = dm.nA + dm.nB;
+  if (dm.kinds & EPIKV_SCORE_BANDZ) {
+    BandRows rows;
+    for (int i = 0; i < kMaxBand; ++i)
+      rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
+    // tokens per CTA: large tiles amortise the extra previous-row read, but
+    // keep at least ~2 CTAs per SM
+    int tpc = 16;
+    while (tpc > 4 && (long)n_seq * nb * ((max_new + tpc - 1) / tpc) < 2L * num_sms) tpc >>= 1;
+    dim3 grid((max_new + tpc - 1) / tpc, nb, n_seq);
+    const int vr = dm.D / 8;
+    if (vr <= kGThreads)
+      bandz_g_kernel<1><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
+    else if (vr <= 2 * kGThreads)
+      bandz_g_kernel<2><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
+    else
+      bandz_g_kernel<4><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
+    ++*launches;
+  }
+  if (dm.kinds & EPIKV_SCORE_LAGKV) {
+    dim3 grid(2 * dm.L, n_seq);
+    const int threads = max(32, (dm.H * dm.d / 8 + 31) / 32 * 32);
+    switch (dm.d / 8) {
+      case 1: lagkv_partial_kernel<1><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      case 2: lagkv_partial_kernel<2><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      case 4: lagkv_partial_kernel<4><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      case 8: lagkv_partial_kernel<8><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      case 16: lagkv_partial_kernel<16><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      default: lagkv_partial_kernel<32><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+    }
+    ++*launches;
+  }
+  {
+    dim3 grid((max_new + kFinTile - 1) / kFinTile, n_seq);
+    const int wmax = max((dm.kinds & EPIKV_SCORE_BANDZ) ? dm.z_window : 1,
+                         (dm.kinds & EPIKV_SCORE_LAGKV) ? dm.lag_window : 1);
+    const int wpl = (wmax + 31) / 32;
+    if (wpl <= 1)
+      score_finalize_kernel<1><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    else if (wpl <= 2)
+      score_finalize_kernel<2><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    else if (wpl <= 4)
+      score_finalize_kernel<4><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    else if (wpl <= 8)
+      score_finalize_kernel<8><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    else
+      score_finalize_kernel<32><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    ++*launches;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace epikv

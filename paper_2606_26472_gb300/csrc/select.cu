@@ -1,0 +1,246 @@
+// Top-K retention under the budget (Sec. 3.1, Sec. 3.3, App. D).
+//
+// One 1024-thread CTA per sequence.  Prefill slots and the trailing recency
+// window R = min(cap, K/4) are always kept; the remaining M = K - P - R slots
+// go to the highest-scoring candidates.  The M-th largest score is found
+// exactly by a 4-pass 8-bit radix select over order-preserving u32 keys
+// (NaN lowest, -0 == +0); candidates above the threshold are kept, and of the
+// candidates equal to it the lowest slots are kept.  Two block-wide ordered
+// scans emit the kept list in ascending slot order.  The slot metadata
+// (scores of every kind and positions) is then compacted in place, which is
+// safe in increasing order because kept[i] >= i.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace epikv {
+
+constexpr int kSelThreads = 1024;
+
+__device__ __forceinline__ uint32_t order_key(float f) {
+  if (f != f) return 0u;          // NaN below every number
+  if (f == 0.0f) f = 0.0f;        // -0 == +0
+  const uint32_t b = __float_as_uint(f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Exclusive prefix sum over the block; *total receives the sum.
+__device__ __forceinline__ int block_exclusive_scan(int v, int* total, int* sh /*[32]*/) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < (kSelThreads / 32) ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    sh[lane] = w;  // inclusive warp totals
+  }
+  __syncthreads();
+  const int before = (warp > 0 ? sh[warp - 1] : 0) + x - v;
+  *total = sh[kSelThreads / 32 - 1];
+  __syncthreads();
+  return before;
+}
+
+__device__ __forceinline__ int block_min(int v, int* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < (kSelThreads / 32) ? sh[lane] : INT_MAX;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) w = min(w, __shfl_xor_sync(0xffffffffu, w, o));
+    if (lane == 0) sh[0] = w;
+  }
+  __syncthreads();
+  const int r = sh[0];
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims dm,
+                                                             const int32_t* __restrict__ seq_ids,
+                                                             const int32_t* __restrict__ budget,
+                                                             const int32_t* __restrict__ trigger,
+                                                             int32_t* __restrict__ kept_out, int kept_stride,
+                                                             int32_t* __restrict__ n_kept_out) {
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int seq = seq_ids[b];
+  if (seq < 0 || seq >= dm.S) {
+    if (tid == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int n = st.n_cache[seq];
+  const int K = budget[b];
+  if (K < 1 || K > dm.T) {
+    if (tid == 0) {
+      set_error(st.err, EPIKV_DEV_BUDGET);
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const int trig = trigger ? trigger[b] : K;
+  if (n <= K || n <= trig) {  // nothing to evict
+    if (tid == 0) {
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const int P = min(st.prefill[seq], n);
+  const int R = min(min(dm.recency_cap, K / 4), max(0, K - P));
+  const int M = max(0, K - P - R);
+  const int c0 = P, c1 = n - R;  // candidates [c0, c1)
+  if (max(K, P) > kept_stride) {
+    if (tid == 0) {
+      set_error(st.err, EPIKV_DEV_KEPT);
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const int kind = st.policy[seq] == EPIKV_SCORE_LAGKV ? 1 : 0;
+  const float* __restrict__ sc = st.score[kind] + (size_t)seq * dm.T;
+  int32_t* out = kept_out + (size_t)b * kept_stride;
+
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sh_prefix, sh_mask, sh_remaining;
+  __shared__ int sh_scan[32];
+
+  // ---- radix select of the M-th largest key among the candidates
+  uint32_t theta = 0xFFFFFFFFu;
+  int need_eq = 0;
+  if (M > 0) {
+    if (tid == 0) { sh_prefix = 0u; sh_mask = 0u; sh_remaining = (uint32_t)M; }
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      if (tid < 256) hist[tid] = 0u;
+      __syncthreads();
+      const uint32_t prefix = sh_prefix, mask = sh_mask;
+      for (int i = c0 + tid; i < c1; i += kSelThreads) {
+        const uint32_t k = order_key(sc[i]);
+        if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (tid < 32) {
+        // lane l owns digits 255-8l .. 248-8l (descending)
+        const int lane = tid;
+        uint32_t lsum = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) lsum += hist[255 - 8 * lane - j];
+        uint32_t incl = lsum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const uint32_t rem = sh_remaining;
+        const unsigned hit = __ballot_sync(0xffffffffu, incl >= rem);
+        const int owner = __ffs(hit) - 1;  // first lane reaching the target
+        if (lane == owner) {
+          uint32_t before = incl - lsum;
+          for (int j = 0; j < 8; ++j) {
+            const int dg = 255 - 8 * lane - j;
+            if (before + hist[dg] >= rem) {
+              sh_prefix = prefix | ((uint32_t)dg << shift);
+              sh_mask = mask | (255u << shift);
+              sh_remaining = rem - before;
+              break;
+            }
+            before += hist[dg];
+          }
+        }
+      }
+      __syncthreads();
+    }
+    theta = sh_prefix;
+    need_eq = (int)sh_remaining;
+  }
+
+  // ---- ordered scans over contiguous per-thread slot ranges
+  const int per = (n + kSelThreads - 1) / kSelThreads;
+  const int a = min(n, tid * per), e = min(n, a + per);
+  int eq_local = 0;
+  for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (order_key(sc[i]) == theta);
+  int tot;
+  const int eq_base = block_exclusive_scan(eq_local, &tot, sh_scan);
+
+  int keep_local = 0, first_ev = INT_MAX;
+  {
+    int eqs = eq_base;
+    for (int i = a; i < e; ++i) {
+      bool keep = (i < c0) || (i >= c1);
+      if (!keep) {
+        const uint32_t k = order_key(sc[i]);
+        keep = k > theta || (k == theta && eqs++ < need_eq);
+      }
+      if (keep) ++keep_local; else first_ev = min(first_ev, i);
+    }
+  }
+  int n_kept;
+  const int keep_base = block_exclusive_scan(keep_local, &n_kept, sh_scan);
+  {
+    int eqs = eq_base, o = keep_base;
+    for (int i = a; i < e; ++i) {
+      bool keep = (i < c0) || (i >= c1);
+      if (!keep) {
+        const uint32_t k = order_key(sc[i]);
+        keep = k > theta || (k == theta && eqs++ < need_eq);
+      }
+      if (keep) out[o++] = i;
+    }
+  }
+  const int fe = min(block_min(first_ev, sh_scan), n_kept);
+  __syncthreads();  // kept list visible to the whole block
+
+  // ---- compact slot metadata in place (kept[i] >= i, increasing i)
+  float* s0 = st.score[0] ? st.score[0] + (size_t)seq * dm.T : nullptr;
+  float* s1 = st.score[1] ? st.score[1] + (size_t)seq * dm.T : nullptr;
+  int32_t* ps = st.pos + (size_t)seq * dm.T;
+  for (int j0 = fe; j0 < n_kept; j0 += kSelThreads) {
+    const int j = j0 + tid;
+    float v0 = 0.f, v1 = 0.f;
+    int32_t p = 0;
+    if (j < n_kept) {
+      const int src = out[j];
+      if (s0) v0 = s0[src];
+      if (s1) v1 = s1[src];
+      p = ps[src];
+    }
+    __syncthreads();
+    if (j < n_kept) {
+      if (s0) s0[j] = v0;
+      if (s1) s1[j] = v1;
+      ps[j] = p;
+    }
+    __syncthreads();
+  }
+  if (tid == 0) {
+    st.n_cache[seq] = n_kept;
+    st.first_changed[seq] = fe;
+    if (n_kept_out) n_kept_out[b] = n_kept;
+    atomicAdd(&st.stats[1], 1ull);
+    atomicAdd(&st.stats[2], (unsigned long long)(n_kept - fe));
+  }
+}
+
+cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
+                          const int32_t* budget, const int32_t* trigger, int32_t* kept, int kept_stride,
+                          int32_t* n_kept, cudaStream_t stream, int* launches) {
+  if (n_seq == 0) return cudaSuccess;
+  select_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride, n_kept);
+  ++*launches;
+  return cudaGetLastError();
+}
+
+}  // namespace epikv

@@ -1,0 +1,192 @@
+"""Drives the CUDA library through its C ABI on seeded synthetic traces and
+checks every stage against the fp64 oracle (test infrastructure).
+
+Acceptance rules:
+* scores: |s_gpu - s_ref| <= 1e-4 * max(1, |s_ref|);
+* kept sets: the oracle's selection run on the GPU's own fp32 scores must
+  equal the GPU's kept list exactly; against the oracle's fp64 scores, a slot
+  may differ only if its reference score is within the score tolerance of the
+  M-th candidate's score (a threshold tie);
+* compacted K/V: byte-identical to the generator's rows of the kept positions.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import epikv_oracle as O
+from paper_2606_26472_gb300 import epikv as E
+from paper_2606_26472_gb300.cache import KVCache
+from synth import gen
+from synth.device import DeviceTrace, as_u16
+
+TOL = 1e-4
+KIND_INDEX = {E.EPIKV_SCORE_BANDZ: 0, E.EPIKV_SCORE_LAGKV: 1}
+
+
+def assert_scores_close(gpu, ref, what=""):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    bound = TOL * np.maximum(1.0, np.abs(ref))
+    bad = np.nonzero(~(np.abs(gpu - ref) <= bound))[0]
+    if bad.size:
+        i = bad[0]
+        raise AssertionError(f"{what}: {bad.size} scores out of tolerance, first at {i}: gpu {gpu[i]!r} ref {ref[i]!r}")
+
+
+class OracleTrace:
+    """fp64 oracle scores of one sequence, from the numpy generator's rows."""
+
+    def __init__(self, model, tabs, seq, length, kinds, z_window=64, lag=16, lag_window=64):
+        self.length = length
+        pos = np.arange(length)
+        self.scores = {}
+        if kinds & E.EPIKV_SCORE_BANDZ:
+            seg = gen.segment_index(model, seq, length)
+            ra = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_a]
+            rb = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_b]
+            self.scores[E.EPIKV_SCORE_BANDZ] = O.bandz_scores(ra, rb, z_window)
+        if kinds & E.EPIKV_SCORE_LAGKV:
+            sp = gen.spike_flags(model, seq, length)
+            K = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0, pos, sp))
+            V = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 1, pos, sp))
+            self.scores[E.EPIKV_SCORE_LAGKV] = O.lagkv_scores(K, V, lag, w=lag_window)
+
+
+class Session:
+    """One context + K/V pool driven call by call from the host."""
+
+    def __init__(self, model, *, n_seq, kinds, layout, max_tokens, max_new, prefill, policies,
+                 z_window=64, lag=16, lag_window=64, recency_cap=128, block_size=16, shuffle_blocks=True,
+                 device="cuda"):
+        self.m = model
+        self.n_seq = n_seq
+        self.kinds = kinds
+        self.prefill = list(prefill)
+        self.policies = list(policies)
+        self.recency_cap = recency_cap
+        self.max_new = max_new
+        self.dt = DeviceTrace(model, device)
+        self.cfg = E.make_config(max_seqs=n_seq, max_cache_tokens=max_tokens, max_new_tokens=max_new,
+                                 num_layers=model.num_layers, num_kv_heads=model.num_kv_heads,
+                                 head_dim=model.head_dim, hidden=model.hidden, n_band_a=len(model.band_a),
+                                 n_band_b=len(model.band_b), z_window=z_window, lag=lag, lag_window=lag_window,
+                                 recency_cap=recency_cap, score_kinds=kinds)
+        nbytes = E.epikv_workspace_bytes(self.cfg)
+        assert nbytes > 0
+        self.ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        self.ctx = E.epikv_init(self.cfg, self.ws, nbytes)
+        for b in range(n_seq):
+            E.epikv_seq_reset(self.ctx, b, self.prefill[b], self.policies[b])
+        bt = None
+        if layout == E.EPIKV_LAYOUT_PAGED:
+            mb = (max_tokens + block_size - 1) // block_size
+            perm = gen.block_permutation(model.seed, n_seq * mb) if shuffle_blocks else np.arange(n_seq * mb)
+            bt = perm.reshape(n_seq, mb)
+        self.cache = KVCache(layout, model.num_layers, model.num_kv_heads, model.head_dim, max_seqs=n_seq,
+                             max_tokens=max_tokens, block_size=block_size, block_table=bt, device=device)
+        self.bt_host = None if bt is None else np.asarray(bt)
+        # canary fill: any row the library wrongly writes or reads stands out
+        self.cache.k.view(torch.int16).fill_(0x7FC1)
+        self.cache.v.view(torch.int16).fill_(0x7FC2)
+        self.kv = self.cache.view()
+        nb = len(model.band_a) + len(model.band_b)
+        self.hid = torch.empty((nb, n_seq * max_new, model.hidden), dtype=torch.bfloat16, device=device) \
+            if kinds & E.EPIKV_SCORE_BANDZ else None
+        self.n_cache = [0] * n_seq
+        self.n_seen = [0] * n_seq
+        self.kept = torch.empty((n_seq, max_tokens), dtype=torch.int32, device=device)
+        self.n_kept = torch.empty((n_seq,), dtype=torch.int32, device=device)
+
+    # ---------------------------------------------------------------- inputs
+    def append(self, entries):
+        """Generate the new tokens' K/V into the cache and their band rows into
+        the packed staging buffer; return (seq_ids, cu_new, max_new, hidden view)."""
+        cu = [0]
+        for b, n in entries:
+            assert self.n_cache[b] + n <= self.cache.T
+            self.dt.kv(b, self.n_seen[b], n, self.n_cache[b], self.cache.k, self.cache.v,
+                       **self.cache.synth_kwargs())
+            if self.hid is not None:
+                for i, layer in enumerate(self.m.band_layers):
+                    out = self.hid[i, cu[-1]:cu[-1] + n]
+                    self.dt.hidden(b, layer, self.n_seen[b], n, out, self.m.hidden)
+            cu.append(cu[-1] + n)
+        seq_ids = torch.tensor([b for b, _ in entries], dtype=torch.int32, device=self.ws.device)
+        cu_new = torch.tensor(cu, dtype=torch.int32, device=self.ws.device)
+        hv = None
+        if self.hid is not None:
+            hv = E.hidden_view([self.hid[i] for i in range(self.hid.shape[0])], self.m.hidden)
+        mx = max([n for _, n in entries] + [0])
+        return seq_ids, cu_new, mx, hv
+
+    def score_update(self, entries):
+        seq_ids, cu_new, mx, hv = self.append(entries)
+        E.epikv_score_update(self.ctx, len(entries), seq_ids, cu_new, mx, hv, self.kv)
+        for b, n in entries:
+            self.n_cache[b] += n
+            self.n_seen[b] += n
+        self._keep_alive = (seq_ids, cu_new)
+
+    def read(self, b, kind):
+        pos, sc, n = E.epikv_read_slots(self.ctx, b, kind, self.cache.T)
+        assert n == self.n_cache[b], (n, self.n_cache[b])
+        return np.array(pos, dtype=np.int64), np.array(sc, dtype=np.float32)
+
+    def select(self, seqs, budgets, triggers=None):
+        seq_ids = torch.tensor(seqs, dtype=torch.int32, device=self.ws.device)
+        bud = torch.tensor(budgets, dtype=torch.int32, device=self.ws.device)
+        trig = None if triggers is None else torch.tensor(triggers, dtype=torch.int32, device=self.ws.device)
+        E.epikv_select(self.ctx, len(seqs), seq_ids, bud, trig, self.kept, self.kept.shape[1], self.n_kept)
+        torch.cuda.synchronize()
+        nk = self.n_kept[:len(seqs)].cpu().numpy()
+        kept = self.kept[:len(seqs)].cpu().numpy()
+        self._sel = (seq_ids,)
+        out = {}
+        for i, b in enumerate(seqs):
+            if nk[i] < self.n_cache[b]:
+                out[b] = kept[i, :nk[i]].astype(np.int64)
+            self.n_cache[b] = int(nk[i])
+        return out
+
+    def compact(self, seqs):
+        seq_ids = self._sel[0]
+        E.epikv_compact(self.ctx, len(seqs), seq_ids, self.kept, self.kept.shape[1], self.kv)
+
+    def error(self):
+        return E.epikv_get_error(self.ctx)
+
+    def cache_rows_u16(self, b, slots):
+        k = as_u16(self.cache.rows(0, b, slots, self.bt_host))
+        v = as_u16(self.cache.rows(1, b, slots, self.bt_host))
+        return k, v
+
+    def close(self):
+        E.epikv_destroy(self.ctx)
+
+
+def check_selection(kept_gpu, pos_pre, sc_gpu_pre, sc_ref_pre, K, P, cap):
+    """Exact check on the GPU's own scores + threshold-tie check on fp64."""
+    exp = O.select_kept(sc_gpu_pre.astype(np.float64), K, P, cap)
+    assert list(kept_gpu) == exp, "selection differs from the oracle run on the GPU's scores"
+    ref = O.select_kept(sc_ref_pre, K, P, cap)
+    if list(kept_gpu) != ref:
+        n = len(sc_ref_pre)
+        Pp = min(P, n)
+        R = min(min(cap, K // 4), max(0, K - Pp))
+        M = max(0, K - Pp - R)
+        cand = sorted(range(Pp, n - R), key=lambda i: (np.isnan(sc_ref_pre[i]), -sc_ref_pre[i], i))
+        theta = sc_ref_pre[cand[M - 1]] if M > 0 else np.inf
+        diff = set(kept_gpu) ^ set(ref)
+        for i in diff:
+            assert abs(sc_ref_pre[i] - theta) <= TOL * max(1.0, abs(theta)), \
+                f"slot {i} differs from the fp64 selection away from the threshold"
+
+
+def check_compaction(sess, b, pos_after):
+    """Compacted rows of every layer and head equal the generator's rows."""
+    sp = gen.spike_flags(sess.m, b, int(pos_after.max()) + 1)
+    tabs = sess.dt.tabs
+    k, v = sess.cache_rows_u16(b, np.arange(len(pos_after)))
+    np.testing.assert_array_equal(k, gen.kv_rows(sess.m, tabs, b, 0, pos_after, sp))
+    np.testing.assert_array_equal(v, gen.kv_rows(sess.m, tabs, b, 1, pos_after, sp))
