@@ -204,6 +204,32 @@ epikv_status epikv_get_stats(epikv_ctx* ctx, epikv_stats* out);
  * in *code (may be NULL); the word is cleared. */
 epikv_status epikv_get_error(epikv_ctx* ctx, int32_t* code);
 
+/* Lag-KV scores of positions 0..n-1 of one sequence, in one call that needs
+ * no context and no device memory beyond its arguments.  The paper has no
+ * counterpart to this entry point: it is for callers that cannot allocate
+ * device memory -- a plugin inside an application whose memory pool owns the
+ * whole GPU, an embedded caller without a device allocator, or a loop that
+ * must never block on cudaMalloc -- and so cannot create the workspace that
+ * epikv_init needs.  It gives the same scores epikv_score_update gives for
+ * the same tokens of a fresh sequence.
+ *   kv         the caller's cache; slots 0..n-1 of `seq` hold positions 0..n-1
+ *   L, H, d    layers, KV heads, head dim (d a power of two in [8, 256],
+ *              H <= 32, H*d/8 <= 256)
+ *   lag, lag_eps, window   as in epikv_config
+ *   d_scores   device float [n]: the output
+ * Working memory is a fixed 2 MiB array inside the library (every GPU that
+ * loads the library holds it until the process exits), so n * 2 * L must not
+ * exceed 524,288 (n <= 8,192 at L = 32): larger requests return EPIKV_EINVAL
+ * and launch nothing.  The first call on each device looks the array's
+ * address up (with that device current); make that first call before any
+ * stream capture.  All calls share the array: calls that overlap on the GPU
+ * (unordered streams) race and must be avoided; calls ordered on one stream
+ * are independent. */
+epikv_status epikv_lagkv_score_noalloc(const epikv_kv_view* kv, int32_t seq, int32_t n,
+                                       int32_t num_layers, int32_t num_kv_heads, int32_t head_dim,
+                                       int32_t lag, float lag_eps, int32_t window, float* d_scores,
+                                       cudaStream_t stream);
+
 void epikv_destroy(epikv_ctx* ctx);
 const char* epikv_status_string(epikv_status s);
 

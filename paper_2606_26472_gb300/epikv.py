@@ -57,6 +57,8 @@ _SIGS = {
     "epikv_read_slots": (C.c_int, [_P, _I, _I, _P, _P, _I, C.POINTER(_I)]),
     "epikv_get_stats": (C.c_int, [_P, C.POINTER(epikv_stats)]),
     "epikv_get_error": (C.c_int, [_P, C.POINTER(_I)]),
+    "epikv_lagkv_score_noalloc": (C.c_int, [C.POINTER(epikv_kv_view), _I, _I, _I, _I, _I, _I, C.c_float, _I,
+                                            _P, _P]),
     "epikv_destroy": (None, [_P]),
     "epikv_status_string": (C.c_char_p, [C.c_int]),
 }
@@ -200,6 +202,13 @@ def epikv_get_error(ctx):
     code = C.c_int32()
     st = load().epikv_get_error(ctx, C.byref(code))
     return st, code.value
+
+
+def epikv_lagkv_score_noalloc(kv, seq, n, num_layers, num_kv_heads, head_dim, lag, lag_eps, window, scores,
+                              stream=None):
+    """Lag-KV scores of positions 0..n-1 of `seq` without any workspace (see epikv.h)."""
+    _check(load().epikv_lagkv_score_noalloc(C.byref(kv), seq, n, num_layers, num_kv_heads, head_dim, lag, lag_eps,
+                                            window, _ptr(scores), _stream(stream)), "epikv_lagkv_score_noalloc")
 
 
 def epikv_destroy(ctx):
