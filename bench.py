@@ -51,6 +51,10 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=20)
+    # a scaled-down variant of the same workload, for profiler captures
+    p.add_argument("--sequences", type=int, default=32)
+    p.add_argument("--budget", type=int, default=8192)
+    p.add_argument("--chunk", type=int, default=128)
     return p.parse_args()
 
 
@@ -67,8 +71,9 @@ def measured_hbm_peak():
 
 
 def ncu_traffic(kernel):
-    """Per-launch DRAM bytes from the committed ncu summary, or None when the
-    kernel's source changed since the counters were taken."""
+    """ncu DRAM traffic of a launch as a ratio to its algorithmic bytes, from
+    the committed summary, or None when the kernel's source changed since the
+    counters were taken."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
@@ -224,7 +229,10 @@ def run_ours(args):
 
     wl = W.config(3)
     m = wl.model
-    Bn, K, C = wl.n_seq, wl.budgets[0], wl.chunk
+    Bn, K, C = args.sequences, args.budget, args.chunk
+    assert K % wl.block_size == 0 and C % wl.block_size == 0
+    workload = WORKLOAD if (Bn, K, C) == (wl.n_seq, wl.budgets[0], wl.chunk) else \
+        f"batch{Bn}_lagkv_paged16_K{K}_chunk{C}"
     L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
     bs = wl.block_size
     T_cap = K + C
@@ -381,12 +389,13 @@ def run_ours(args):
         return
     peak, peak_src = measured_hbm_peak()
     ach = compact_bytes / args.steps / (t_compact / args.steps / 1e3) / 1e9
-    traffic = ncu_traffic("compact_kernel")
+    ratio = ncu_traffic("compact_kernel")
+    traffic = None if ratio is None else ratio * compact_bytes / args.steps
     line = {
         "metric": METRIC, "value": world * tokens / (ms / 1e3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "sequences": Bn, "context": 32768, "budget_K": K, "chunk": C,
+        "config": {"workload": workload, "sequences": Bn, "context": 32768, "budget_K": K, "chunk": C,
                    "layers": L, "kv_heads": H, "head_dim": d, "kv_dtype": "bf16", "layout": "paged16_shuffled",
                    "score": "lagkv_lag16_w64", "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
@@ -401,7 +410,7 @@ def run_ours(args):
         "clocks": clk,
         "e2e": e2e,
     }
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and workload == WORKLOAD:
         line["cpu_baseline"] = cpu_baseline()
     print(json.dumps(line), flush=True)
     if world > 1:
