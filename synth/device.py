@@ -28,6 +28,15 @@ def load():
         lib.synth_kv.argtypes = [C.c_uint64, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                  C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int64,
                                  C.c_int64, C.c_int64, C.c_int64, C.c_void_p, C.c_int, C.c_int, C.c_void_p]
+        lib.synth_hidden_batch.restype = C.c_int
+        lib.synth_hidden_batch.argtypes = [C.c_uint64, C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_int, C.c_float,
+                                           C.c_float, C.c_float, C.c_float, C.c_void_p, C.c_void_p, C.c_int64,
+                                           C.c_void_p, C.c_int64, C.c_void_p]
+        lib.synth_kv_batch.restype = C.c_int
+        lib.synth_kv_batch.argtypes = [C.c_uint64, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int,
+                                       C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int,
+                                       C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_void_p, C.c_int, C.c_int,
+                                       C.c_void_p]
         _lib = lib
     return _lib
 
@@ -79,6 +88,40 @@ class DeviceTrace:
                             _stream(stream))
         if r != 0:
             raise RuntimeError(f"synth_kv failed ({r})")
+
+
+class DeviceBatchTrace(DeviceTrace):
+    """DeviceTrace plus batched generation for ragged decode steps: every row
+    of a step in one launch per layer (hidden) or one launch (K/V)."""
+
+    def __init__(self, model, n_seq, max_len, device="cuda"):
+        super().__init__(model, device)
+        seg = np.stack([gen.segment_index(model, b, max_len) for b in range(n_seq)])
+        self.seg_tab = torch.from_numpy(seg).to(device)
+        self.seg_stride = max_len
+
+    def hidden_batch(self, layer, seqs, pos, out, row_stride, stream=None):
+        m, tb = self.m, self.tabs
+        r = load().synth_hidden_batch(m.seed & 0xFFFFFFFFFFFFFFFF, layer, seqs.numel(), seqs.data_ptr(),
+                                      pos.data_ptr(), m.hidden, float(tb.scale[layer]), float(tb.drift[layer]),
+                                      float(tb.seg_amp[layer]), float(gen.INV_SD), self.mean[layer].data_ptr(),
+                                      self.seg_tab.data_ptr(), self.seg_stride,
+                                      out if isinstance(out, int) else out.data_ptr(), row_stride, _stream(stream))
+        if r != 0:
+            raise RuntimeError(f"synth_hidden_batch failed ({r})")
+
+    def kv_batch(self, seqs, pos, slots, k, v, *, layout, stride_layer, stride_seq=0, stride_block=0, stride_token,
+                 block_table=None, max_blocks=0, block_size=0, stream=None):
+        m = self.m
+        r = load().synth_kv_batch(m.seed & 0xFFFFFFFFFFFFFFFF, seqs.numel(), seqs.data_ptr(), pos.data_ptr(),
+                                  slots.data_ptr(), m.num_layers, m.num_kv_heads, m.head_dim, m.spike_per_10k,
+                                  self.kv_scale.data_ptr(), self.kv_off.data_ptr(),
+                                  k if isinstance(k, int) else k.data_ptr(), v if isinstance(v, int) else v.data_ptr(),
+                                  layout, stride_layer, stride_seq, stride_block, stride_token,
+                                  None if block_table is None else block_table.data_ptr(), max_blocks, block_size,
+                                  _stream(stream))
+        if r != 0:
+            raise RuntimeError(f"synth_kv_batch failed ({r})")
 
 
 def as_u16(t: torch.Tensor) -> np.ndarray:

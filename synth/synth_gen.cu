@@ -116,6 +116,79 @@ __global__ void kv_kernel(uint64_t seed, int seq, int pos0, int n, int slot0, in
   *reinterpret_cast<uint4*>(vw.base[kind] + (row + h * d + j0) * 2) = q;
 }
 
+// Batched rows: row i is (seqs[i], pos[i]); seg is [n_seq][seg_stride].
+__global__ void hidden_batch_kernel(uint64_t seed, int layer, int n, const int32_t* __restrict__ seqs,
+                                    const int32_t* __restrict__ poss, int D, float scale, float drift,
+                                    float seg_amp, float inv_sd, const float* __restrict__ mean,
+                                    const int32_t* __restrict__ seg, int64_t seg_stride, uint16_t* __restrict__ out,
+                                    int64_t row_stride) {
+  const int t = blockIdx.x;
+  if (t >= n) return;
+  const int seq = seqs[t], pos = poss[t];
+  const uint64_t key = row_key(S_HIDDEN, seed, (uint64_t)seq, (uint64_t)layer, 0, (uint64_t)pos);
+  const float tf = __fmul_rn((float)pos, 1.52587890625e-05f);
+  const float c = __fmul_rn(__fmul_rn(scale, __fadd_rn(1.0f, __fmul_rn(drift, tf))), inv_sd);
+  const bool has_seg = seg_amp != 0.0f;
+  const float bamp = __fmul_rn(seg_amp, inv_sd);
+  const uint64_t skey =
+      has_seg ? row_key(S_SEGMENT, seed, (uint64_t)seq, (uint64_t)layer, 0, (uint64_t)seg[seq * seg_stride + pos]) : 0;
+  uint16_t* row = out + (int64_t)t * row_stride;
+  for (int v = threadIdx.x; v < D / 8; v += blockDim.x) {
+    float f[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int j = v * 8 + e;
+      float x = __fmul_rn(normal16(mix64(key + (uint64_t)j)), c);
+      if (has_seg) x = __fadd_rn(x, __fmul_rn(normal16(mix64(skey + (uint64_t)j)), bamp));
+      f[e] = __fadd_rn(x, mean[j]);
+    }
+    uint4 q;
+    q.x = pack2(f[0], f[1]);
+    q.y = pack2(f[2], f[3]);
+    q.z = pack2(f[4], f[5]);
+    q.w = pack2(f[6], f[7]);
+    *reinterpret_cast<uint4*>(row + v * 8) = q;
+  }
+}
+
+// grid (n rows, L, 2); row i = (seqs[i], pos[i]) written to slot slots[i].
+__global__ void kv_batch_kernel(uint64_t seed, int n, const int32_t* __restrict__ seqs,
+                                const int32_t* __restrict__ poss, const int32_t* __restrict__ slots, int L, int H,
+                                int d, int spike_per_10k, const float* __restrict__ kv_scale,
+                                const float* __restrict__ kv_off, View vw) {
+  const int t = blockIdx.x, layer = blockIdx.y, kind = blockIdx.z;
+  const int lpt = d / 8;
+  const int h = threadIdx.x / lpt, j0 = (threadIdx.x % lpt) * 8;
+  if (t >= n || h >= H) return;
+  const int seq = seqs[t], pos = poss[t], slot = slots[t];
+  const uint64_t sp = row_key(S_SPIKE, seed, (uint64_t)seq, 0, 0, (uint64_t)pos);
+  const bool spike = pos >= 1 && (sp % 10000ull) < (uint64_t)spike_per_10k;
+  const float cs = __fmul_rn(kv_scale[(kind * L + layer) * H + h], spike ? 4.0f : 1.0f);
+  const uint64_t key = row_key(kind == 0 ? S_KEY : S_VALUE, seed, (uint64_t)seq, (uint64_t)layer, (uint64_t)h,
+                               (uint64_t)pos);
+  const float* off = kv_off + ((int64_t)(kind * L + layer) * H + h) * d;
+  float f[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int j = j0 + e;
+    f[e] = __fadd_rn(__fmul_rn(normal16(mix64(key + (uint64_t)j)), cs), off[j]);
+  }
+  int64_t row;
+  if (vw.layout == 0) {
+    row = (int64_t)layer * vw.stride_layer + (int64_t)seq * vw.stride_seq + (int64_t)slot * vw.stride_token;
+  } else {
+    const int blk = vw.block_table[(int64_t)seq * vw.max_blocks + slot / vw.block_size];
+    row = (int64_t)layer * vw.stride_layer + (int64_t)blk * vw.stride_block +
+          (int64_t)(slot % vw.block_size) * vw.stride_token;
+  }
+  uint4 q;
+  q.x = pack2(f[0], f[1]);
+  q.y = pack2(f[2], f[3]);
+  q.z = pack2(f[4], f[5]);
+  q.w = pack2(f[6], f[7]);
+  *reinterpret_cast<uint4*>(vw.base[kind] + (row + h * d + j0) * 2) = q;
+}
+
 }  // namespace
 
 extern "C" {
@@ -152,6 +225,43 @@ int synth_kv(uint64_t seed, int seq, int pos0, int n, int slot0, int L, int H, i
   dim3 grid(n, L, 2);
   const int threads = (H * d / 8 + 31) / 32 * 32;
   kv_kernel<<<grid, threads, 0, stream>>>(seed, seq, pos0, n, slot0, L, H, d, spike_per_10k, d_kv_scale, d_kv_off, vw);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+// Batched hidden rows of one layer: row i of d_out is (d_seqs[i], d_pos[i]).
+int synth_hidden_batch(uint64_t seed, int layer, int n, const int32_t* d_seqs, const int32_t* d_pos, int D,
+                       float scale, float drift, float seg_amp, float inv_sd, const float* d_mean,
+                       const int32_t* d_seg, int64_t seg_stride, void* d_out, int64_t row_stride,
+                       cudaStream_t stream) {
+  if (n <= 0) return 0;
+  if (D % 8 || !d_mean || !d_out || !d_seqs || !d_pos || (seg_amp != 0.0f && !d_seg)) return 1;
+  hidden_batch_kernel<<<n, 256, 0, stream>>>(seed, layer, n, d_seqs, d_pos, D, scale, drift, seg_amp, inv_sd, d_mean,
+                                            d_seg, seg_stride, static_cast<uint16_t*>(d_out), row_stride);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+// Batched K/V rows: (d_seqs[i], d_pos[i]) written to slot d_slots[i] of sequence d_seqs[i].
+int synth_kv_batch(uint64_t seed, int n, const int32_t* d_seqs, const int32_t* d_pos, const int32_t* d_slots, int L,
+                   int H, int d, int spike_per_10k, const float* d_kv_scale, const float* d_kv_off, void* k, void* v,
+                   int layout, int64_t stride_layer, int64_t stride_seq, int64_t stride_block, int64_t stride_token,
+                   const int32_t* block_table, int max_blocks, int block_size, cudaStream_t stream) {
+  if (n <= 0) return 0;
+  if (d % 8 || H * d / 8 > 1024 || !k || !v || !d_seqs || !d_pos || !d_slots) return 1;
+  View vw;
+  vw.base[0] = static_cast<char*>(k);
+  vw.base[1] = static_cast<char*>(v);
+  vw.layout = layout;
+  vw.stride_layer = stride_layer;
+  vw.stride_seq = stride_seq;
+  vw.stride_block = stride_block;
+  vw.stride_token = stride_token;
+  vw.block_table = block_table;
+  vw.max_blocks = max_blocks;
+  vw.block_size = block_size;
+  dim3 grid(n, L, 2);
+  const int threads = (H * d / 8 + 31) / 32 * 32;
+  kv_batch_kernel<<<grid, threads, 0, stream>>>(seed, n, d_seqs, d_pos, d_slots, L, H, d, spike_per_10k, d_kv_scale,
+                                                d_kv_off, vw);
   return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }
 

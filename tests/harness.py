@@ -128,6 +128,19 @@ class Session:
             self.n_seen[b] += n
         self._keep_alive = (seq_ids, cu_new)
 
+    def step(self, entries, budgets, triggers):
+        """One epikv_step (score + device trigger + select + compact)."""
+        seq_ids, cu_new, mx, hv = self.append(entries)
+        n = len(entries)
+        bud = torch.tensor(budgets, dtype=torch.int32, device=self.ws.device)
+        trig = torch.tensor(triggers, dtype=torch.int32, device=self.ws.device)
+        out = torch.empty(n, dtype=torch.int32, device=self.ws.device)
+        E.epikv_step(self.ctx, n, seq_ids, cu_new, mx, bud, trig, hv, self.kv, out)
+        lens = out.cpu().numpy()
+        for i, (b, k) in enumerate(entries):
+            self.n_seen[b] += k
+            self.n_cache[b] = int(lens[i])
+
     def read(self, b, kind):
         pos, sc, n = E.epikv_read_slots(self.ctx, b, kind, self.cache.T)
         assert n == self.n_cache[b], (n, self.n_cache[b])
@@ -181,6 +194,50 @@ def check_selection(kept_gpu, pos_pre, sc_gpu_pre, sc_ref_pre, K, P, cap):
         for i in diff:
             assert abs(sc_ref_pre[i] - theta) <= TOL * max(1.0, abs(theta)), \
                 f"slot {i} differs from the fp64 selection away from the threshold"
+
+
+def oracle_bandz_at(model, tabs, seq, t, w=64):
+    """fp64 EpiKV score of position t from the generator's rows of its window."""
+    if t == 0:
+        return 0.0
+    lo = max(0, t - w)
+    pos = np.arange(lo, t + 1)
+    seg = gen.segment_index(model, seq, t + 1)
+    z = {}
+    for l in model.band_layers:
+        rows = gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg))
+        g = [O.hidden_change(rows[i - 1], rows[i]) for i in range(1, len(pos))]   # positions lo+1 .. t
+        window = g[-min(w, t):]
+        z[l] = [O.window_zscore(window)]
+    return float(O.epiphany_score([z[l] for l in model.band_a], [z[l] for l in model.band_b])[0])
+
+
+def oracle_lag_at(model, tabs, seq, t, lag=16, w=64):
+    """fp64 Lag-KV score of position t from the generator's rows it depends on."""
+    t0 = max(0, t - w + 1)
+    first = max(0, (t0 // lag - 1) * lag)
+    pos = np.arange(first, t + 1)
+    sp = gen.spike_flags(model, seq, t + 1)
+    K = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0, pos, sp))
+    V = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 1, pos, sp))
+    u = []
+    for tt in range(t0, t + 1):
+        c = tt // lag
+        if c == 0:
+            u.append(0.0)
+        else:
+            lo = (c - 1) * lag - first
+            u.append(O.lag_token_variance(K[tt - first], V[tt - first], K[lo:lo + lag], V[lo:lo + lag]))
+    return float(O.rolling_mean(np.array(u), w)[-1])
+
+
+def check_compaction_sampled(sess, b, pos_after, n_rows, rng):
+    """Compacted rows at `n_rows` random slots (every layer, head, K and V)."""
+    slots = np.sort(rng.choice(len(pos_after), size=min(n_rows, len(pos_after)), replace=False))
+    sp = gen.spike_flags(sess.m, b, int(pos_after.max()) + 1)
+    k, v = sess.cache_rows_u16(b, slots)
+    np.testing.assert_array_equal(k, gen.kv_rows(sess.m, sess.dt.tabs, b, 0, pos_after[slots], sp))
+    np.testing.assert_array_equal(v, gen.kv_rows(sess.m, sess.dt.tabs, b, 1, pos_after[slots], sp))
 
 
 def check_compaction(sess, b, pos_after):
