@@ -109,7 +109,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   // issue the loads of the batch at cursor c into stage s
   auto issue = [&](const Cursor& c, int s) {
     const int nrows = min(rpb, c.end - c.i);
-    char* kvb = kv.base[c.kvk];
+    char* kvb = c.kvk ? kv.base[1] : kv.base[0];
     unsigned char* stage = smem + s * kStageBytes;
     const int32_t* kl = kept + (size_t)c.b * kept_stride;
     const char* src[kMaxRowsPerLane];

@@ -125,10 +125,43 @@ __global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm
   }
 }
 
-constexpr int kLagBatch = 16;
+constexpr int kLagSeg = 16;     // tokens per segment (never crosses a chunk boundary)
+constexpr int kLagOffs = 256;   // slot offsets looked up per group of tokens
 
-// grid: (2L (layer, K|V), batch entries); block: max(32, H*d/8) threads,
-// lanes-per-head LH = d/8 consecutive threads own one head (8 channels each).
+__device__ __forceinline__ uint32_t bf16x2_min(uint32_t a, uint32_t b) {
+  __nv_bfloat162 r = __hmin2(*reinterpret_cast<__nv_bfloat162*>(&a), *reinterpret_cast<__nv_bfloat162*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+__device__ __forceinline__ uint32_t bf16x2_max(uint32_t a, uint32_t b) {
+  __nv_bfloat162 r = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&a), *reinterpret_cast<__nv_bfloat162*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+__device__ __forceinline__ uint4 q_min(const uint4& a, const uint4& b) {
+  return make_uint4(bf16x2_min(a.x, b.x), bf16x2_min(a.y, b.y), bf16x2_min(a.z, b.z), bf16x2_min(a.w, b.w));
+}
+__device__ __forceinline__ uint4 q_max(const uint4& a, const uint4& b) {
+  return make_uint4(bf16x2_max(a.x, b.x), bf16x2_max(a.y, b.y), bf16x2_max(a.z, b.z), bf16x2_max(a.w, b.w));
+}
+
+// Minimum and reciprocal range denominator of the previous chunk, per channel.
+__device__ __forceinline__ void prev_range(const uint4& pmn, const uint4& pmx, float eps, float (&mn)[8],
+                                           float (&inv)[8]) {
+  float mx[8];
+  unpack8(pmn, mn);
+  unpack8(pmx, mx);
+#pragma unroll
+  for (int e = 0; e < 8; ++e) inv[e] = 1.f / (mx[e] - mn[e] + eps);
+}
+
+// grid: (2L (layer, K|V), batch entries); block: max(32, H*d/8) threads;
+// LH = d/8 consecutive lanes own one head, 8 channels each.
+//
+// Tokens are taken in segments that stay inside one chunk: every token of a
+// segment is normalised with the same previous-chunk range, so the segment's
+// reductions are independent of one another.  Chunk ranges (min, max) are
+// bf16 values and are kept packed (exact).  The variance of a token's head
+// is taken from the moments of y = x~ - 1/2 (x~ in [0, 1] inside the range),
+// one two-value group reduction per token.
 template <int LH>
 __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
                                                              const int32_t* __restrict__ seq_ids,
@@ -155,105 +188,101 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
   const int ch = h * dm.d + q * 8;  // first channel of this thread within the token row
   __nv_bfloat16* rng = st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd;
 
-  float pmn[8], pmx[8], cmn[8], cmx[8], inv[8];
+  uint4 pmn = make_uint4(0, 0, 0, 0), pmx = pmn, cmn = pmn, cmx = pmn;
   if (active) {
-    unpack8(*reinterpret_cast<const uint4*>(rng + 0 * hd + ch), pmn);
-    unpack8(*reinterpret_cast<const uint4*>(rng + 1 * hd + ch), pmx);
-    unpack8(*reinterpret_cast<const uint4*>(rng + 2 * hd + ch), cmn);
-    unpack8(*reinterpret_cast<const uint4*>(rng + 3 * hd + ch), cmx);
-  } else {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) pmn[e] = pmx[e] = cmn[e] = cmx[e] = 0.f;
+    pmn = *reinterpret_cast<const uint4*>(rng + 0 * hd + ch);
+    pmx = *reinterpret_cast<const uint4*>(rng + 1 * hd + ch);
+    cmn = *reinterpret_cast<const uint4*>(rng + 2 * hd + ch);
+    cmx = *reinterpret_cast<const uint4*>(rng + 3 * hd + ch);
   }
-#pragma unroll
-  for (int e = 0; e < 8; ++e) inv[e] = 1.f / (pmx[e] - pmn[e] + dm.lag_eps);
+  float mn[8], inv[8];
+  prev_range(pmn, pmx, dm.lag_eps, mn, inv);
 
   const float inv_d = 1.f / (float)dm.d;
-  const char* kvbase = kv.base[kvk];
-  __shared__ float hv[kLagBatch][32];  // per token, per head (the host admits H <= 32)
+  const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
+  __shared__ int64_t soff[kLagOffs];
+  __shared__ float hv[2][kLagSeg][32];  // [segment parity][token][head]; the host admits H <= 32
   float* part = st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L);
+  int r = p0 % dm.lag;                   // position of the next token inside its chunk
+  int parity = 0;
 
-  for (int i0 = 0; i0 < n_new; i0 += kLagBatch) {
-    const int nbt = min(kLagBatch, n_new - i0);
-    uint4 x[kLagBatch];
+  for (int g0 = 0; g0 < n_new; g0 += kLagOffs) {
+    const int gn = min(kLagOffs, n_new - g0);
+    __syncthreads();
+    for (int t = tid; t < gn; t += blockDim.x) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
+    __syncthreads();
+    for (int i = 0; i < gn;) {
+      const int seg = min(min(dm.lag - r, gn - i), kLagSeg);
+      const bool has_prev = p0 + g0 + i >= dm.lag;   // the segment's chunk is not chunk 0
+      uint4 x[kLagSeg];
 #pragma unroll
-    for (int j = 0; j < kLagBatch; ++j) {
-      x[j] = make_uint4(0, 0, 0, 0);
-      if (j < nbt && active) {
-        const int64_t off = kv_row_offset(kv, layer, seq, nc0 + i0 + j, dm.T);
-        if (off >= 0)
-          x[j] = ld_stream16(kvbase + (off + ch) * 2);
-        else
-          set_error(st.err, EPIKV_DEV_SLOT);
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < kLagBatch; ++j) {
-      if (j < nbt) {
-        const int pos = p0 + i0 + j;
-        const int c = pos / dm.lag;
-        const int r = pos - c * dm.lag;
-        float xf[8];
-        unpack8(x[j], xf);
-        float var = 0.f;
-        if (c >= 1) {  // uniform across the block: every thread sees the same token
-          float xn[8], s = 0.f;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            xn[e] = (xf[e] - pmn[e]) * inv[e];
-            s += xn[e];
-          }
-          const float mean = group_sum(s, LH) * inv_d;
-          float ss = 0.f;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float dv = xn[e] - mean;
-            ss = fmaf(dv, dv, ss);
-          }
-          var = group_sum(ss, LH) * inv_d;
-        }
-        if (q == 0 && active) hv[j][h] = var;
-        if (r == 0) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) cmn[e] = cmx[e] = xf[e];
-        } else {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            cmn[e] = fminf(cmn[e], xf[e]);
-            cmx[e] = fmaxf(cmx[e], xf[e]);
-          }
-        }
-        if (r == dm.lag - 1) {  // chunk complete: it becomes the previous chunk
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            pmn[e] = cmn[e];
-            pmx[e] = cmx[e];
-            inv[e] = 1.f / (pmx[e] - pmn[e] + dm.lag_eps);
-          }
+      for (int j = 0; j < kLagSeg; ++j) {
+        x[j] = make_uint4(0, 0, 0, 0);
+        if (j < seg && active) {
+          const int64_t off = soff[i + j];
+          if (off >= 0)
+            x[j] = ld_stream16(kvbase + (off + ch) * 2);
+          else
+            set_error(st.err, EPIKV_DEV_SLOT);
         }
       }
+#pragma unroll
+      for (int j = 0; j < kLagSeg; ++j) {
+        if (j < seg) {
+          float var = 0.f;
+          if (has_prev) {  // uniform across the block
+            float xf[8], s1 = 0.f, s2 = 0.f;
+            unpack8(x[j], xf);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float y = fmaf(xf[e] - mn[e], inv[e], -0.5f);
+              s1 += y;
+              s2 = fmaf(y, y, s2);
+            }
+#pragma unroll
+            for (int o = LH >> 1; o > 0; o >>= 1) {
+              s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+              s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+            }
+            const float mean = s1 * inv_d;
+            var = fmaxf(fmaf(-mean, mean, s2 * inv_d), 0.f);
+          }
+          if (q == 0 && active) hv[parity][j][h] = var;
+        }
+      }
+      // advance the running range of the current chunk
+      if (r == 0) {
+        cmn = x[0];
+        cmx = x[0];
+      }
+#pragma unroll
+      for (int j = 0; j < kLagSeg; ++j)
+        if (j < seg) {
+          cmn = q_min(cmn, x[j]);
+          cmx = q_max(cmx, x[j]);
+        }
+      __syncthreads();
+      if (tid < seg) {
+        float sum = 0.f;
+        for (int hh = 0; hh < dm.H; ++hh) sum += hv[parity][tid][hh];
+        part[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+      }
+      parity ^= 1;
+      r += seg;
+      if (r == dm.lag) {  // chunk complete: it becomes the previous chunk
+        pmn = cmn;
+        pmx = cmx;
+        prev_range(pmn, pmx, dm.lag_eps, mn, inv);
+        r = 0;
+      }
+      i += seg;
     }
-    __syncthreads();
-    if (tid < nbt) {
-      float s = 0.f;
-      for (int hh = 0; hh < dm.H; ++hh) s += hv[tid][hh];
-      part[(size_t)(i0 + tid) * (2 * dm.L) + blockIdx.x] = s;
-    }
-    __syncthreads();
   }
   if (active) {
-    auto pack = [](const float* f) {
-      uint4 q4;
-      q4.x = (__float_as_uint(f[0]) >> 16) | (__float_as_uint(f[1]) & 0xFFFF0000u);
-      q4.y = (__float_as_uint(f[2]) >> 16) | (__float_as_uint(f[3]) & 0xFFFF0000u);
-      q4.z = (__float_as_uint(f[4]) >> 16) | (__float_as_uint(f[5]) & 0xFFFF0000u);
-      q4.w = (__float_as_uint(f[6]) >> 16) | (__float_as_uint(f[7]) & 0xFFFF0000u);
-      return q4;  // exact: every value is a bf16 value held in fp32
-    };
-    *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = pack(pmn);
-    *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = pack(pmx);
-    *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = pack(cmn);
-    *reinterpret_cast<uint4*>(rng + 3 * hd + ch) = pack(cmx);
+    *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = pmn;
+    *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = pmx;
+    *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = cmn;
+    *reinterpret_cast<uint4*>(rng + 3 * hd + ch) = cmx;
   }
 }
 
