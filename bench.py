@@ -329,7 +329,8 @@ def run_ours(args):
     assert st_ == E.EPIKV_OK, f"device error {code}"
     t_score = sum(p[0].elapsed_time(p[1]) for p in phase)
     t_select = sum(p[1].elapsed_time(p[2]) for p in phase)
-    t_compact = sum(p[2].elapsed_time(p[3]) for p in phase)
+    per_compact = sorted(p[2].elapsed_time(p[3]) for p in phase)
+    t_compact = sum(per_compact)
     rows_moved = stats1["rows_moved"] - stats0["rows_moved"]
     tokens = stats1["tokens_scored"] - stats0["tokens_scored"]
     assert tokens == Bn * C * args.steps
@@ -402,6 +403,7 @@ def run_ours(args):
         "compaction_gbs": ach,
         "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
                                 "compact": t_compact / args.steps},
+        "compact_ms_min_median_max": [per_compact[0], per_compact[len(per_compact) // 2], per_compact[-1]],
         "step_hbm_gbs": (compact_bytes + score_bytes) / (ms / 1e3) / 1e9,
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src,

@@ -101,15 +101,34 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                :: "r"(smem_u32(bar)), "r"(bytes) : "memory");
 }
 
-// One probe (the hardware may suspend the thread for up to ~1 us); true when
-// the phase with `parity` has completed.
+#ifndef EPIKV_MBAR_SPIN
+#define EPIKV_MBAR_SPIN 2
+#endif
+
+// One probe; true when the phase with `parity` has completed.  The default
+// (2) may suspend the thread for a short, hardware-chosen time; 1 polls
+// without suspending; 0 asks for a suspension of up to 1 us.
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
+#if EPIKV_MBAR_SPIN == 1
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+#elif EPIKV_MBAR_SPIN == 2
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+#else
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, 1000;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+#endif
   return ok != 0;
 }
 

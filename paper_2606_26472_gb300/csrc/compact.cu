@@ -18,12 +18,32 @@
 
 namespace epikv {
 
-constexpr int kStageBytes = 16384;
-constexpr int kStages = 4;
+#ifndef EPIKV_COMPACT_STAGE_BYTES
+#define EPIKV_COMPACT_STAGE_BYTES 16384
+#endif
+#ifndef EPIKV_COMPACT_STAGES
+#define EPIKV_COMPACT_STAGES 4
+#endif
+#ifndef EPIKV_COMPACT_CTAS_PER_SM
+#define EPIKV_COMPACT_CTAS_PER_SM 2  // more CTAs per SM overload the memory system (measured)
+#endif
+#ifndef EPIKV_COMPACT_ORDER
+#define EPIKV_COMPACT_ORDER 0  // 0: units sequence-major, 1: layer-major
+#endif
+#ifndef EPIKV_COMPACT_HEAD_SPLIT
+#define EPIKV_COMPACT_HEAD_SPLIT 0  // 0: chosen on the device to fill the grid
+#endif
+constexpr int kStageBytes = EPIKV_COMPACT_STAGE_BYTES;
+constexpr int kStages = EPIKV_COMPACT_STAGES;
 constexpr int kMaxRowsPerLane = 4;
 constexpr int kMaxRPB = 32 * kMaxRowsPerLane;
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s: far beyond any real copy
 constexpr uint64_t kDrainNs = 100000000ull;   // 0.1 s per stage after a timeout
+
+#ifndef EPIKV_COMPACT_STAGED_BLOCKS
+#define EPIKV_COMPACT_STAGED_BLOCKS 1024  // block-table entries kept in shared memory (larger tables: global reads)
+#endif
+constexpr int kStagedBlocks = EPIKV_COMPACT_STAGED_BLOCKS;
 
 struct Cursor {
   int u;      // unit index (this CTA strides by gridDim.x)
@@ -40,6 +60,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   __shared__ char* dptr[kStages][kMaxRPB];
   __shared__ int stage_rows[kStages];
   int* list = reinterpret_cast<int*>(smem + kStages * kStageBytes);
+  int* bt_s = list + (n_seq + 31) / 32 * 32;  // the current sequence's block table
   const int lane = threadIdx.x;
 
   // ---- the batch entries that evicted (every CTA builds the same list)
@@ -58,24 +79,22 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   __syncwarp();
   if (n_ev == 0) return;
 
-  // ---- head split: the one (1, 2, 4, ...) whose unit count fills the grid best
+  // ---- head split: whole token rows unless too few streams evict to give
+  // every CTA one (small TMA copies cost much more per byte than a tail)
   const int G = gridDim.x;
   int hs = 1;
-  {
-    double best = -1.0;
-    for (int c = 1; c <= dm.H; c <<= 1) {
-      if (dm.H % c != 0 || (dm.H / c) * dm.d * 2 < 256) break;
-      const long units = (long)n_ev * 2 * dm.L * c;
-      const long rounds = (units + G - 1) / G;
-      const double eff = (double)units / (double)(rounds * G);
-      if (eff > best + 1e-3) { best = eff; hs = c; }
-    }
+  if (EPIKV_COMPACT_HEAD_SPLIT > 0 && dm.H % EPIKV_COMPACT_HEAD_SPLIT == 0) {
+    hs = EPIKV_COMPACT_HEAD_SPLIT;
+  } else {
+    while ((long)n_ev * 2 * dm.L * hs < G && dm.H % (2 * hs) == 0 && (dm.H / (2 * hs)) * dm.d * 2 >= 256) hs *= 2;
   }
   const int rb = (dm.H / hs) * dm.d * 2;               // bytes per row piece
   const int64_t piece_elems = (int64_t)(dm.H / hs) * dm.d;
   const int rpb = min(kStageBytes / rb, kMaxRPB);      // rows per batch
   const int upe = 2 * dm.L * hs;
   const int units = n_ev * upe;
+  const bool paged = kv.layout == EPIKV_LAYOUT_PAGED;
+  const bool bt_in_smem = paged && kv.max_blocks <= kStagedBlocks;
 
   if (lane == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
@@ -86,7 +105,14 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
 
   auto load_unit = [&](Cursor& c) {
     while (c.u < units) {
-      const int e = c.u / upe, rem = c.u % upe;
+      int e, rem;
+      if (EPIKV_COMPACT_ORDER == 1) {
+        e = c.u % n_ev;
+        rem = c.u / n_ev;
+      } else {
+        e = c.u / upe;
+        rem = c.u % upe;
+      }
       c.layer = rem / (2 * hs);
       c.kvk = (rem / hs) & 1;
       c.hg = rem % hs;
@@ -105,13 +131,41 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       load_unit(c);
     }
   };
+  // kept slots of the batch at c, one load per row, issued early and used later
+  auto prefetch = [&](const Cursor& c, int (&pk)[kMaxRowsPerLane]) {
+    if (c.u >= units) return;
+    const int nrows = min(rpb, c.end - c.i);
+    const int32_t* kl = kept + (size_t)c.b * kept_stride + c.i;
+#pragma unroll
+    for (int j = 0; j < kMaxRowsPerLane; ++j) {
+      const int r = lane + 32 * j;
+      pk[j] = r < nrows ? __ldg(kl + r) : 0;
+    }
+  };
+  int staged_seq = -1;
+  // element offset of a slot of the current sequence, -1 outside the view
+  auto slot_offset = [&](int layer, int seq, int slot) -> int64_t {
+    if (!bt_in_smem) return kv_row_offset(kv, layer, seq, slot, dm.T);
+    if (slot < 0) return -1;
+    const int bi = slot / kv.block_size;
+    if (bi >= kv.max_blocks) return -1;
+    const int blk = bt_s[bi];
+    if (blk < 0 || blk >= kv.num_blocks) return -1;
+    return (int64_t)layer * kv.stride_layer + (int64_t)blk * kv.stride_block +
+           (int64_t)(slot - bi * kv.block_size) * kv.stride_token;
+  };
 
-  // issue the loads of the batch at cursor c into stage s
-  auto issue = [&](const Cursor& c, int s) {
+  // issue the loads of the batch at cursor c (kept slots pk) into stage s
+  auto issue = [&](const Cursor& c, const int (&pk)[kMaxRowsPerLane], int s) {
+    if (bt_in_smem && c.seq != staged_seq) {
+      __syncwarp();
+      for (int j = lane; j < kv.max_blocks; j += 32) bt_s[j] = __ldg(kv.block_table + (int64_t)c.seq * kv.max_blocks + j);
+      __syncwarp();
+      staged_seq = c.seq;
+    }
     const int nrows = min(rpb, c.end - c.i);
     char* kvb = c.kvk ? kv.base[1] : kv.base[0];
     unsigned char* stage = smem + s * kStageBytes;
-    const int32_t* kl = kept + (size_t)c.b * kept_stride;
     const char* src[kMaxRowsPerLane];
     uint32_t total = 0;
 #pragma unroll
@@ -121,9 +175,9 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       bool ok = false;
       if (r < nrows) {
         const int i = c.i + r;
-        const int from = kl[i];
-        const int64_t so = from >= i ? kv_row_offset(kv, c.layer, c.seq, from, dm.T) : -1;
-        const int64_t dof = kv_row_offset(kv, c.layer, c.seq, i, dm.T);
+        const int from = pk[j];
+        const int64_t so = from >= i ? slot_offset(c.layer, c.seq, from) : -1;
+        const int64_t dof = slot_offset(c.layer, c.seq, i);
         ok = so >= 0 && dof >= 0;
         if (ok) {
           src[j] = kvb + (so + c.hg * piece_elems) * 2;
@@ -148,12 +202,15 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   Cursor ld;
   ld.u = blockIdx.x;
   load_unit(ld);
+  int pk[kMaxRowsPerLane];
+  prefetch(ld, pk);
   int k_issue = 0, k_store = 0;
   bool timed_out = false;
   for (int p = 0; p < kStages - 1 && ld.u < units; ++p) {
-    issue(ld, k_issue % kStages);
+    issue(ld, pk, k_issue % kStages);
     ++k_issue;
     advance(ld);
+    prefetch(ld, pk);
   }
   while (k_store < k_issue) {
     const int s = k_store % kStages;
@@ -171,9 +228,10 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
     if (ld.u < units) {
       tma_wait_read<1>();  // the stage about to be refilled has been read out
       __syncwarp();
-      issue(ld, k_issue % kStages);
+      issue(ld, pk, k_issue % kStages);
       ++k_issue;
       advance(ld);
+      prefetch(ld, pk);    // its latency hides behind the next barrier wait
     }
   }
   if (timed_out) {
@@ -188,7 +246,8 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
 static int g_ctas_per_sm = 0;
 
 static size_t compact_smem(int n_seq) {
-  return (size_t)kStages * kStageBytes + (size_t)((n_seq + 31) / 32 * 32) * sizeof(int);
+  return (size_t)kStages * kStageBytes + (size_t)((n_seq + 31) / 32 * 32) * sizeof(int) +
+         (size_t)kStagedBlocks * sizeof(int);
 }
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm) {
@@ -200,6 +259,7 @@ cudaError_t compact_prepare(int device, int* ctas_per_sm) {
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, 32, compact_smem(64));
   if (e != cudaSuccess) return e;
   g_ctas_per_sm = n > 0 ? n : 1;
+  if (EPIKV_COMPACT_CTAS_PER_SM > 0 && EPIKV_COMPACT_CTAS_PER_SM < g_ctas_per_sm) g_ctas_per_sm = EPIKV_COMPACT_CTAS_PER_SM;
   if (ctas_per_sm) *ctas_per_sm = g_ctas_per_sm;
   return cudaSuccess;
 }
