@@ -55,6 +55,9 @@ def parse():
     p.add_argument("--sequences", type=int, default=32)
     p.add_argument("--budget", type=int, default=8192)
     p.add_argument("--chunk", type=int, default=128)
+    # the band-z kernels' workload: the 2,048-token single-sequence case, one
+    # fresh sequence per step (reported for the per-kernel rooflines)
+    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k"])
     return p.parse_args()
 
 
@@ -424,10 +427,111 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_bandz2k(args):
+    """One step = a fresh sequence: its 2,048 tokens scored with the band-z
+    score (15 band layers of 4096 bf16), the cache cut to K = 512, all 32
+    layers' K/V compacted -- epikv_step on one sequence.  Each step's
+    sequence has its own resident cache and hidden rows."""
+    import torch
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    from paper_2606_26472_gb300.cache import KVCache
+    from synth import workloads as W
+    from synth.device import DeviceTrace
+
+    rank, local_rank, world = dist_env()
+    assert world == 1, "the band-z workload is a single-GPU measurement"
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+    wl = W.config(1)
+    m = wl.model
+    T, K = wl.max_len, wl.budgets[0]
+    S = args.warmup + args.steps
+    nb = len(m.band_layers)
+    dt = DeviceTrace(m, dev)
+    cache = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, m.num_layers, m.num_kv_heads, m.head_dim, max_seqs=S, max_tokens=T,
+                    device=dev)
+    hid = torch.empty((nb, S, T, m.hidden), dtype=torch.bfloat16, device=dev)
+    for s_ in range(S):
+        dt.kv(s_, 0, T, 0, cache.k, cache.v, **cache.synth_kwargs())
+        for i, layer in enumerate(m.band_layers):
+            dt.hidden(s_, layer, 0, T, hid[i, s_], m.hidden)
+    cfg = E.make_config(max_seqs=S, max_cache_tokens=T, max_new_tokens=T, n_band_a=len(m.band_a),
+                        n_band_b=len(m.band_b), score_kinds=E.EPIKV_SCORE_BANDZ)
+    ws = torch.empty(E.epikv_workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws.numel())
+    kv = cache.view()
+    views = [E.hidden_view([hid[i, s_] for i in range(nb)], m.hidden) for s_ in range(S)]
+    ids = [torch.tensor([s_], dtype=torch.int32, device=dev) for s_ in range(S)]
+    cu = torch.tensor([0, T], dtype=torch.int32, device=dev)
+    budget = torch.tensor([K], dtype=torch.int32, device=dev)
+    trigger = torch.tensor([K], dtype=torch.int32, device=dev)
+    n_out = torch.empty(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(s_):
+        E.epikv_seq_reset(ctx, s_, 0, E.EPIKV_SCORE_BANDZ)
+        E.epikv_step(ctx, 1, ids[s_], cu, T, budget, trigger, views[s_], kv, n_out)
+
+    for s_ in range(args.warmup):
+        step(s_)
+    torch.cuda.synchronize()
+    stats0 = E.epikv_get_stats(ctx)
+    phase = []
+    for _ in range(args.steps):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        for e in evs:
+            e.record(stream)
+        phase.append(evs)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for i in range(args.steps):
+        E.epikv_set_phase_events(ctx, phase[i])
+        step(args.warmup + i)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    E.epikv_set_phase_events(ctx, None)
+    ms = t0.elapsed_time(t1)
+    stats1 = E.epikv_get_stats(ctx)
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    tokens = stats1["tokens_scored"] - stats0["tokens_scored"]
+    rows = stats1["rows_moved"] - stats0["rows_moved"]
+    t_score = sum(p[0].elapsed_time(p[1]) for p in phase) / args.steps
+    t_select = sum(p[1].elapsed_time(p[2]) for p in phase) / args.steps
+    t_compact = sum(p[2].elapsed_time(p[3]) for p in phase) / args.steps
+    score_bytes = T * nb * m.hidden * 2 + 2 * nb * m.hidden * 2       # rows + h_prev write/read
+    compact_bytes = 2 * rows / args.steps * m.num_layers * 2 * m.num_kv_heads * m.head_dim * 2
+    peak, peak_src = measured_hbm_peak()
+    g = score_bytes / (t_score / 1e3) / 1e9
+    c = compact_bytes / (t_compact / 1e3) / 1e9
+    line = {"metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "single_2k_bandz_K512_fresh_sequence_per_step", "band_layers": nb,
+                       "hidden": m.hidden, "budget_K": K, "layout": "contiguous",
+                       "l2": "inputs larger than L2 (%.1f GiB resident)" % ((cache.k.numel() * 2 + hid.numel()) * 2 / 2 ** 30)},
+            "kernels_ms_per_step": {"score": t_score, "select": t_select, "compact": t_compact},
+            "score_phase_gbs": g, "compaction_gbs": c,
+            "roofline": {"bound": "hbm", "kernel": "score phase (bandz_g_kernel + score_finalize_kernel)",
+                         "achieved": g, "peak": peak, "unit": "GB/s", "frac": g / peak, "peak_source": peak_src,
+                         "traffic": None, "algorithmic_bytes_per_launch": score_bytes},
+            "gpu_launches": 5 * args.steps}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload == "bandz2k":
+        run_bandz2k(args)
     else:
         run_ours(args)
 

@@ -83,11 +83,11 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   // every CTA one (small TMA copies cost much more per byte than a tail)
   const int G = gridDim.x;
   int hs = 1;
-  if (EPIKV_COMPACT_HEAD_SPLIT > 0 && dm.H % EPIKV_COMPACT_HEAD_SPLIT == 0) {
-    hs = EPIKV_COMPACT_HEAD_SPLIT;
-  } else {
-    while ((long)n_ev * 2 * dm.L * hs < G && dm.H % (2 * hs) == 0 && (dm.H / (2 * hs)) * dm.d * 2 >= 256) hs *= 2;
-  }
+#if EPIKV_COMPACT_HEAD_SPLIT > 0
+  if (dm.H % EPIKV_COMPACT_HEAD_SPLIT == 0) hs = EPIKV_COMPACT_HEAD_SPLIT;
+#else
+  while ((long)n_ev * 2 * dm.L * hs < G && dm.H % (2 * hs) == 0 && (dm.H / (2 * hs)) * dm.d * 2 >= 256) hs *= 2;
+#endif
   const int rb = (dm.H / hs) * dm.d * 2;               // bytes per row piece
   const int64_t piece_elems = (int64_t)(dm.H / hs) * dm.d;
   const int rpb = min(kStageBytes / rb, kMaxRPB);      // rows per batch

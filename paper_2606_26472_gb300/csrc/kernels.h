@@ -21,6 +21,7 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
                            cudaStream_t stream, int* launches);
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm);
+cudaError_t finalize_prepare();
 
 cudaError_t launch_reset_seq(const DevState& st, const Dims& dm, int seq, int prefill, int policy,
                              cudaStream_t stream);

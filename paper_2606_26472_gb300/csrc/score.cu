@@ -23,6 +23,7 @@ namespace epikv {
 
 constexpr int kGThreads = 256;
 constexpr int kGUnroll = 4;
+constexpr int kMaxTokPerCta = 16;
 
 struct BandRows {
   const __nv_bfloat16* p[kMaxBand];
@@ -65,7 +66,7 @@ __global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm
     prev[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
   }
 
-  __shared__ float red[kGUnroll][kGThreads / 32];
+  __shared__ float red[kMaxTokPerCta][kGThreads / 32];  // per token of the tile, per warp
   for (int t = t0; t < t1; t += kGUnroll) {
     uint4 cur[kGUnroll][VPT];
 #pragma unroll
@@ -77,7 +78,6 @@ __global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm
         cur[u][k] = (t + u < t1 && v < VR) ? ld_stream16(row + v * 8) : make_uint4(0, 0, 0, 0);
       }
     }
-    float part[kGUnroll];
 #pragma unroll
     for (int u = 0; u < kGUnroll; ++u) {
       float acc = 0.f;
@@ -92,11 +92,8 @@ __global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm
           acc = fmaf(dlt, dlt, acc);
         }
       }
-      part[u] = warp_sum(acc);
-    }
-    if (lane == 0) {
-#pragma unroll
-      for (int u = 0; u < kGUnroll; ++u) red[u][warp] = part[u];
+      acc = warp_sum(acc);
+      if (lane == 0 && t + u < t1) red[t - t0 + u][warp] = acc;
     }
     // the last valid row of this group is the previous row of the next group
     const int last = min(kGUnroll, t1 - t) - 1;
@@ -106,15 +103,14 @@ __global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm
 #pragma unroll
         for (int k = 0; k < VPT; ++k) prev[k] = cur[u][k];
       }
-    __syncthreads();
-    if (tid < kGUnroll && t + tid < t1) {
-      float s = 0.f;
+  }
+  __syncthreads();
+  if (tid < t1 - t0) {
+    float s = 0.f;
 #pragma unroll
-      for (int w = 0; w < kGThreads / 32; ++w) s += red[tid][w];
-      const int pos = p0 + t + tid;
-      if (pos >= 1) ring[pos & (dm.G - 1)] = sqrtf(s);
-    }
-    __syncthreads();
+    for (int w = 0; w < kGThreads / 32; ++w) s += red[tid][w];
+    const int pos = p0 + t0 + tid;
+    if (pos >= 1) ring[pos & (dm.G - 1)] = sqrtf(s);
   }
   if (t1 == n_new) {
 #pragma unroll
@@ -319,40 +315,47 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
       if (lane == 0) st.pos[(size_t)seq * dm.T + nc0 + i] = pos;
     }
     if (dm.kinds & EPIKV_SCORE_BANDZ) {
-      for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
+      // every g value the tile's windows reach, all band layers, one round of loads
+      extern __shared__ float sg[];  // [nb][span]
+      const int span = kFinTile + dm.z_window - 1;
+      const int pos_base = p0 + i_lo - (dm.z_window - 1);  // position held by sg[band][0]
+      const int pos_end = p0 + i_hi;
+      for (int idx = tid; idx < nb * span; idx += kFinThreads) {
+        const int band = idx / span;
+        const int pos = pos_base + (idx - band * span);
+        sg[idx] = (pos >= 1 && pos < pos_end) ? st.g_ring[((size_t)seq * nb + band) * dm.G + (pos & Gm)] : 0.f;
+      }
+      __syncthreads();
+      // a lane per (token, band layer): lpt lanes per token, 32/lpt tokens per warp
+      const int lpt = nb <= 16 ? 16 : 32;
+      const int sub = lane / lpt, band = lane % lpt;
+      for (int i0 = i_lo + warp * (32 / lpt); i0 < i_hi; i0 += kFinThreads / lpt) {
+        const int i = i0 + sub;
         const int pos = p0 + i;
-        float s = 0.f;
-        if (pos >= 1) {
+        const bool live = i < i_hi && pos >= 1 && band < nb;
+        float za = 0.f, zb = 0.f;
+        if (live) {
           const int n = min(dm.z_window, pos);
-          const float inv_n = 1.f / (float)n;
-          float za = 0.f, zb = 0.f;
-          for (int band = 0; band < nb; ++band) {
-            const float* ring = st.g_ring + ((size_t)seq * nb + band) * dm.G;
-            const float gnew = ring[pos & Gm];
-            float v[WPL], dsum = 0.f;
-#pragma unroll
-            for (int m = 0; m < WPL; ++m) {
-              const int k = lane + 32 * m;  // window offset: position pos - k
-              v[m] = k < n ? ring[(pos - k) & Gm] - gnew : 0.f;
-              dsum += v[m];
-            }
-            const float mean_d = warp_sum(dsum) * inv_n;
-            float dev = 0.f;
-#pragma unroll
-            for (int m = 0; m < WPL; ++m) {
-              const int k = lane + 32 * m;
-              if (k < n) {
-                const float e = v[m] - mean_d;
-                dev = fmaf(e, e, dev);
-              }
-            }
-            const float sigma = sqrtf(warp_sum(dev) * inv_n);
-            const float z = -mean_d / (sigma + dm.z_eps);  // g(t) - mu = -(mean of g - g(t))
-            if (band < dm.nA) za += z; else zb += z;
+          const float* row = sg + band * span + (pos - pos_base);   // row[-k] = g at position pos - k
+          const float gnew = row[0];
+          float dsum = 0.f;
+          for (int k = 0; k < n; ++k) dsum += row[-k] - gnew;
+          const float mean_d = dsum / (float)n;
+          float dev = 0.f;
+          for (int k = 0; k < n; ++k) {
+            const float e = (row[-k] - gnew) - mean_d;
+            dev = fmaf(e, e, dev);
           }
-          s = za / (float)dm.nA - zb / (float)dm.nB;
+          const float sigma = sqrtf(dev / (float)n);
+          const float z = -mean_d / (sigma + dm.z_eps);  // g(t) - mu = -(mean of g - g(t))
+          if (band < dm.nA) za = z; else zb = z;
         }
-        if (lane == 0) st.score[0][(size_t)seq * dm.T + nc0 + i] = s;
+        for (int o = lpt >> 1; o > 0; o >>= 1) {  // stays inside each token's lane group
+          za += __shfl_xor_sync(0xffffffffu, za, o);
+          zb += __shfl_xor_sync(0xffffffffu, zb, o);
+        }
+        if (band == 0 && i < i_hi)
+          st.score[0][(size_t)seq * dm.T + nc0 + i] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
       }
     }
     if (dm.kinds & EPIKV_SCORE_LAGKV) {
@@ -409,6 +412,21 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
 }
 
 // ------------------------------------------------------------------ launchers
+// dynamic shared memory of the finalize kernel: the band windows of a tile
+static size_t finalize_smem(const Dims& dm) {
+  if (!(dm.kinds & EPIKV_SCORE_BANDZ)) return 0;
+  return (size_t)(dm.nA + dm.nB) * (kFinTile + dm.z_window - 1) * sizeof(float);
+}
+
+cudaError_t finalize_prepare() {
+  const int mx = (int)((size_t)kMaxBand * (kFinTile + kMaxWindow - 1) * sizeof(float));
+  cudaError_t e = cudaFuncSetAttribute(score_finalize_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  return e;
+}
 cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
                                 const int32_t* cu_new, int max_new, const epikv_hidden_view* hv,
                                 const KvDev* kv, int num_sms, cudaStream_t stream, int* launches) {
@@ -420,7 +438,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
       rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
     // tokens per CTA: large tiles amortise the extra previous-row read, but
     // keep at least ~2 CTAs per SM
-    int tpc = 16;
+    int tpc = kMaxTokPerCta;
     while (tpc > 4 && (long)n_seq * nb * ((max_new + tpc - 1) / tpc) < 2L * num_sms) tpc >>= 1;
     dim3 grid((max_new + tpc - 1) / tpc, nb, n_seq);
     const int vr = dm.D / 8;
@@ -450,16 +468,17 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
     const int wmax = max((dm.kinds & EPIKV_SCORE_BANDZ) ? dm.z_window : 1,
                          (dm.kinds & EPIKV_SCORE_LAGKV) ? dm.lag_window : 1);
     const int wpl = (wmax + 31) / 32;
+    const size_t smem = finalize_smem(dm);
     if (wpl <= 1)
-      score_finalize_kernel<1><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+      score_finalize_kernel<1><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
     else if (wpl <= 2)
-      score_finalize_kernel<2><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+      score_finalize_kernel<2><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
     else if (wpl <= 4)
-      score_finalize_kernel<4><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+      score_finalize_kernel<4><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
     else if (wpl <= 8)
-      score_finalize_kernel<8><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+      score_finalize_kernel<8><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
     else
-      score_finalize_kernel<32><<<grid, kFinThreads, 0, stream>>>(st, dm, seq_ids, cu_new, max_new);
+      score_finalize_kernel<32><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
     ++*launches;
   }
   return cudaGetLastError();
