@@ -256,7 +256,7 @@ def run_ours(args):
     fresh = C // bs
     n_steps = args.warmup + args.steps
     e2e_steps = 0 if args.no_e2e else args.e2e_steps
-    n_blocks = Bn * common + n_steps * Bn * fresh + (Bn * fresh if e2e_steps else 0)
+    n_blocks = Bn * common + n_steps * Bn * fresh + (2 * Bn * fresh if e2e_steps else 0)
     perm = gen.block_permutation(m.seed ^ rank, Bn * common).reshape(Bn, common)
 
     def table(fresh_base):
@@ -358,29 +358,49 @@ def run_ours(args):
     # ---- end to end: new tokens' K/V from pinned host memory, new lengths back
     e2e = None
     if e2e_steps:
-        tab = table(e2e_base)
-        view = cache.view(tab)
+        # two sets of fresh blocks: step i+1's K/V are copied in on a side
+        # stream while step i runs, as a serving loop would overlap them
+        tabs = [table(e2e_base + j * Bn * fresh) for j in range(2)]
+        views_e = [cache.view(t) for t in tabs]
         n_payload = min(4, e2e_steps)
         payload = torch.empty((n_payload, 2, L, Bn * fresh, bs, H, d), dtype=torch.bfloat16, pin_memory=True)
         pos_base = K + n_steps * C
+        lo = e2e_base
         for j in range(n_payload):
             for b in range(Bn):
-                dt.kv(b, pos_base + j * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tab))
-            payload[j, 0].copy_(cache.k[:, e2e_base:e2e_base + Bn * fresh])
-            payload[j, 1].copy_(cache.v[:, e2e_base:e2e_base + Bn * fresh])
+                dt.kv(b, pos_base + j * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tabs[0]))
+            payload[j, 0].copy_(cache.k[:, lo:lo + Bn * fresh])
+            payload[j, 1].copy_(cache.v[:, lo:lo + Bn * fresh])
         lens = torch.empty((e2e_steps, Bn), dtype=torch.int32, pin_memory=True)
+        copy_stream = torch.cuda.Stream(device=dev)
+        copied = [torch.cuda.Event() for _ in range(e2e_steps)]
+        stepped = [torch.cuda.Event() for _ in range(e2e_steps)]
+
+        def h2d(i):   # step i's new K/V into block set i % 2, after step i-2 released it
+            lo_i = e2e_base + (i % 2) * Bn * fresh
+            with torch.cuda.stream(copy_stream):
+                if i >= 2:
+                    copy_stream.wait_event(stepped[i - 2])
+                src = payload[i % n_payload]
+                for kind, pool in ((0, cache.k), (1, cache.v)):
+                    for l in range(L):
+                        pool[l, lo_i:lo_i + Bn * fresh].copy_(src[kind, l], non_blocking=True)
+                copied[i].record(copy_stream)
+
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
+        copy_stream.wait_event(e0)
+        h2d(0)
         for i in range(e2e_steps):
-            src = payload[i % n_payload]
-            for kind, pool in ((0, cache.k), (1, cache.v)):
-                for l in range(L):
-                    pool[l, e2e_base:e2e_base + Bn * fresh].copy_(src[kind, l], non_blocking=True)
-            step(None, view)
+            if i + 1 < e2e_steps:
+                h2d(i + 1)
+            stream.wait_event(copied[i])
+            step(None, views_e[i % 2])
+            stepped[i].record(stream)
             lens[i].copy_(n_out, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
@@ -388,7 +408,7 @@ def run_ours(args):
         assert (lens.numpy() == K).all()
         e2e = {"value": e_value, "unit": UNIT,
                "h2d_bytes_per_step": int(payload[0].numel() * 2), "d2h_bytes_per_step": Bn * 4,
-               "steps": e2e_steps}
+               "steps": e2e_steps, "overlap": "step i+1's host-to-device copy runs on a side stream during step i"}
         st_, code = E.epikv_get_error(ctx)
         assert st_ == E.EPIKV_OK, f"device error {code} in e2e"
 

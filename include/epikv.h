@@ -144,6 +144,7 @@ epikv_status epikv_seq_reset(epikv_ctx* ctx, int32_t seq, int32_t prefill_len, i
 /* Score the new tokens of a batch and append them to each sequence's slots.
  *   d_seq_ids [n_seq]   device: sequence id of each batch entry
  *   d_cu_new  [n_seq+1] device: prefix offsets of the new tokens per entry
+ *                       (d_cu_new[0] = 0, non-decreasing)
  *   max_new             host: an upper bound of every entry's new tokens
  *                       (<= cfg.max_new_tokens; sizes the grid)
  *   hidden              band rows of the new tokens (needed for BANDZ)

@@ -29,95 +29,137 @@ struct BandRows {
   const __nv_bfloat16* p[kMaxBand];
 };
 
-// grid: (token tiles, band layers, batch entries); block: 256 threads.
+// Persistent grid; block: 256 threads.  The rows of the call, flattened as
+// r = band * total_new + packed_row, are split into gridDim.x equal
+// contiguous shares, so every CTA streams the same number of rows.  A CTA
+// walks its share in runs that stay inside one (band layer, batch entry),
+// 16 tokens at most; the previous row of a run's first token is the last row
+// of the run before it when they are consecutive, else it is loaded (from
+// the saved h_prev for a sequence's first new token).
 template <int VPT>
-__global__ void __launch_bounds__(kGThreads) bandz_g_kernel(DevState st, Dims dm, BandRows rows,
+__global__ void __launch_bounds__(kGThreads, (VPT >= 4 ? 2 : 4)) bandz_g_kernel(DevState st, Dims dm, BandRows rows,
                                                             int64_t row_stride,
                                                             const int32_t* __restrict__ seq_ids,
-                                                            const int32_t* __restrict__ cu_new,
-                                                            int max_new, int tok_per_cta) {
-  const int b = blockIdx.z, band = blockIdx.y;
-  const int seq = seq_ids[b];
-  const int r0 = cu_new[b];
-  const int n_new = cu_new[b + 1] - r0;
-  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
-    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+                                                            const int32_t* __restrict__ cu_new, int n_seq,
+                                                            int max_new) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // the whole batch must be well formed, else nothing is read
+  __shared__ int bad;
+  if (tid == 0) bad = 0;
+  __syncthreads();
+  for (int b = tid; b < n_seq; b += kGThreads) {
+    const int seq = seq_ids[b], n = cu_new[b + 1] - cu_new[b];
+    if (seq < 0 || seq >= dm.S || n < 0 || n > max_new || cu_new[0] != 0) bad = 1;
+  }
+  __syncthreads();
+  if (bad) {
+    if (tid == 0 && blockIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
     return;
   }
-  const int t0 = blockIdx.x * tok_per_cta;
-  if (t0 >= n_new) return;
-  const int t1 = min(t0 + tok_per_cta, n_new);
-  const int p0 = st.n_seen[seq];
-  const int par = st.hp_parity[seq];
   const int nb = dm.nA + dm.nB;
+  const int total = cu_new[n_seq];
+  const int64_t R = (int64_t)nb * total;
+  int64_t r = R * blockIdx.x / gridDim.x;
+  const int64_t r_end = R * (blockIdx.x + 1) / gridDim.x;
+  if (r >= r_end) return;
   const int VR = dm.D >> 3;  // 16-byte vectors per row
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  __shared__ float red[kMaxTokPerCta][kGThreads / 32];  // per token of a run, per warp
 
-  const __nv_bfloat16* hp_rd = st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D;
-  __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
-  const __nv_bfloat16* base = rows.p[band];
-  float* ring = st.g_ring + ((size_t)seq * nb + band) * dm.G;
-
-  const __nv_bfloat16* prow = (t0 == 0) ? hp_rd : base + (int64_t)(r0 + t0 - 1) * row_stride;
-  uint4 prev[VPT];
-#pragma unroll
-  for (int k = 0; k < VPT; ++k) {
-    const int v = tid + k * kGThreads;
-    prev[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
+  int band = (int)(r / total), row = (int)(r - (int64_t)band * total);
+  int b = 0;  // batch entry holding `row` (largest b with cu_new[b] <= row and a token)
+  {
+    int lo = 0, hi = n_seq - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (cu_new[mid] <= row) lo = mid; else hi = mid - 1;
+    }
+    b = lo;
+    while (cu_new[b + 1] <= row) ++b;  // skip empty entries
   }
-
-  __shared__ float red[kMaxTokPerCta][kGThreads / 32];  // per token of the tile, per warp
-  for (int t = t0; t < t1; t += kGUnroll) {
-    uint4 cur[kGUnroll][VPT];
-#pragma unroll
-    for (int u = 0; u < kGUnroll; ++u) {
-      const __nv_bfloat16* row = base + (int64_t)(r0 + t + u) * row_stride;
+  uint4 prev[VPT];
+  int prev_band = -1, prev_row = -1;  // what `prev` holds
+  while (r < r_end) {
+    const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
+    const int seq = seq_ids[b];
+    const int t0 = row - r0;
+    const int len = (int)min((int64_t)min(kMaxTokPerCta, n_new - t0), r_end - r);
+    const int t1 = t0 + len;
+    const int p0 = st.n_seen[seq];
+    const int par = st.hp_parity[seq];
+    const __nv_bfloat16* base = rows.p[band];
+    if (!(prev_band == band && prev_row == row - 1 && t0 > 0)) {
+      const __nv_bfloat16* prow = t0 == 0 ? st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D
+                                          : base + (int64_t)(row - 1) * row_stride;
 #pragma unroll
       for (int k = 0; k < VPT; ++k) {
         const int v = tid + k * kGThreads;
-        cur[u][k] = (t + u < t1 && v < VR) ? ld_stream16(row + v * 8) : make_uint4(0, 0, 0, 0);
+        prev[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
       }
     }
+    for (int t = t0; t < t1; t += kGUnroll) {
+      uint4 cur[kGUnroll][VPT];
 #pragma unroll
-    for (int u = 0; u < kGUnroll; ++u) {
-      float acc = 0.f;
+      for (int u = 0; u < kGUnroll; ++u) {
+        const __nv_bfloat16* rp = base + (int64_t)(r0 + t + u) * row_stride;
 #pragma unroll
-      for (int k = 0; k < VPT; ++k) {
-        float c[8], p[8];
-        unpack8(cur[u][k], c);
-        unpack8(u == 0 ? prev[k] : cur[u - 1][k], p);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float dlt = c[e] - p[e];
-          acc = fmaf(dlt, dlt, acc);
+        for (int k = 0; k < VPT; ++k) {
+          const int v = tid + k * kGThreads;
+          cur[u][k] = (t + u < t1 && v < VR) ? ld_stream16(rp + v * 8) : make_uint4(0, 0, 0, 0);
         }
       }
-      acc = warp_sum(acc);
-      if (lane == 0 && t + u < t1) red[t - t0 + u][warp] = acc;
-    }
-    // the last valid row of this group is the previous row of the next group
-    const int last = min(kGUnroll, t1 - t) - 1;
 #pragma unroll
-    for (int u = 0; u < kGUnroll; ++u)
-      if (u == last) {
+      for (int u = 0; u < kGUnroll; ++u) {
+        float acc = 0.f;
 #pragma unroll
-        for (int k = 0; k < VPT; ++k) prev[k] = cur[u][k];
+        for (int k = 0; k < VPT; ++k) {
+          float c[8], p[8];
+          unpack8(cur[u][k], c);
+          unpack8(u == 0 ? prev[k] : cur[u - 1][k], p);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float dlt = c[e] - p[e];
+            acc = fmaf(dlt, dlt, acc);
+          }
+        }
+        acc = warp_sum(acc);
+        if (lane == 0 && t + u < t1) red[t - t0 + u][warp] = acc;
       }
-  }
-  __syncthreads();
-  if (tid < t1 - t0) {
-    float s = 0.f;
+      // the last valid row of this group is the previous row of the next group
+      const int last = min(kGUnroll, t1 - t) - 1;
 #pragma unroll
-    for (int w = 0; w < kGThreads / 32; ++w) s += red[tid][w];
-    const int pos = p0 + t0 + tid;
-    if (pos >= 1) ring[pos & (dm.G - 1)] = sqrtf(s);
-  }
-  if (t1 == n_new) {
+      for (int u = 0; u < kGUnroll; ++u)
+        if (u == last) {
 #pragma unroll
-    for (int k = 0; k < VPT; ++k) {
-      const int v = tid + k * kGThreads;
-      if (v < VR) *reinterpret_cast<uint4*>(hp_wr + v * 8) = prev[k];
+          for (int k = 0; k < VPT; ++k) prev[k] = cur[u][k];
+        }
     }
+    __syncthreads();
+    if (tid < len) {
+      float sum = 0.f;
+#pragma unroll
+      for (int w = 0; w < kGThreads / 32; ++w) sum += red[tid][w];
+      const int pos = p0 + t0 + tid;
+      if (pos >= 1) st.g_ring[((size_t)seq * nb + band) * dm.G + (pos & (dm.G - 1))] = sqrtf(sum);
+    }
+    if (t1 == n_new) {  // the sequence's last new row of this band is the next call's previous row
+      __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
+#pragma unroll
+      for (int k = 0; k < VPT; ++k) {
+        const int v = tid + k * kGThreads;
+        if (v < VR) *reinterpret_cast<uint4*>(hp_wr + v * 8) = prev[k];
+      }
+    }
+    __syncthreads();  // red is reused by the next run
+    prev_band = band;
+    prev_row = row + len - 1;
+    r += len;
+    row += len;
+    if (row == total) {
+      row = 0;
+      ++band;
+      b = 0;
+    }
+    while (b < n_seq && cu_new[b + 1] <= row) ++b;
   }
 }
 
@@ -436,18 +478,25 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
     BandRows rows;
     for (int i = 0; i < kMaxBand; ++i)
       rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
-    // tokens per CTA: large tiles amortise the extra previous-row read, but
-    // keep at least ~2 CTAs per SM
-    int tpc = kMaxTokPerCta;
-    while (tpc > 4 && (long)n_seq * nb * ((max_new + tpc - 1) / tpc) < 2L * num_sms) tpc >>= 1;
-    dim3 grid((max_new + tpc - 1) / tpc, nb, n_seq);
+    // persistent: as many CTAs as are resident, never more than rows
+    static int resident[3] = {0, 0, 0};
     const int vr = dm.D / 8;
-    if (vr <= kGThreads)
-      bandz_g_kernel<1><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
-    else if (vr <= 2 * kGThreads)
-      bandz_g_kernel<2><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
+    const int vi = vr <= kGThreads ? 0 : vr <= 2 * kGThreads ? 1 : 2;
+    if (!resident[vi]) {
+      int per_sm = 1;
+      if (vi == 0) cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bandz_g_kernel<1>, kGThreads, 0);
+      if (vi == 1) cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bandz_g_kernel<2>, kGThreads, 0);
+      if (vi == 2) cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bandz_g_kernel<4>, kGThreads, 0);
+      resident[vi] = (per_sm > 0 ? per_sm : 1) * num_sms;
+    }
+    const int64_t rows_bound = (int64_t)nb * n_seq * max_new;
+    const int grid = (int)(rows_bound < resident[vi] ? rows_bound : resident[vi]);
+    if (vi == 0)
+      bandz_g_kernel<1><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
+    else if (vi == 1)
+      bandz_g_kernel<2><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
     else
-      bandz_g_kernel<4><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, max_new, tpc);
+      bandz_g_kernel<4><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
     ++*launches;
   }
   if (dm.kinds & EPIKV_SCORE_LAGKV) {
