@@ -30,6 +30,13 @@ R10 Lag-KV: chunks of lag positions at fixed boundaries t = c*lag; token t in
     of chunk c-1; population variance over the head dimension; K and V
     variances are added; the mean is over (layer, head); u(t) = 0 in chunk 0;
     the score is the mean of u over the last min(w, t+1) positions <= t.
+R11 HS-variance (Eq. 2): the rolling mean of g over the same window as the
+    z-score (R2); band means as in R1; s(0) = 0.
+R12 KV-key / KV-val variance: the population variance over the head
+    dimension of the stored key (value) vector of each (layer, head), mean
+    over (layer, head), then the rolling mean of R10; every position has a
+    value (no chunk 0 exception).
+R13 lag-kv-key: Lag-KV (R10) with the key term only.
 """
 from __future__ import annotations
 
@@ -86,6 +93,23 @@ def epiphany_score(z_band_a, z_band_b):
     return za - zb
 
 
+def rolling_band_mean(g, w=64):
+    """g-bar[t]: mean of g over the trailing window of R2 (Eq. 2); 0 at t = 0."""
+    g = np.asarray(g, dtype=np.float64)
+    m = np.zeros(g.shape[0])
+    for t in range(1, g.shape[0]):
+        m[t] = np.mean(g[max(1, t - w + 1): t + 1])
+    return m
+
+
+def hsvar_scores(rows_a, rows_b, w=64):
+    """HS-variance score s(t) = g-bar_A(t) - g-bar_B(t) (Eq. 2, Tab. 1,
+    reading R11) of every position of one sequence."""
+    ma = [rolling_band_mean(hidden_change_trace(r), w) for r in rows_a]
+    mb = [rolling_band_mean(hidden_change_trace(r), w) for r in rows_b]
+    return np.mean(ma, axis=0) - np.mean(mb, axis=0)
+
+
 def bandz_scores(rows_a, rows_b, w=64, eps=Z_EPS):
     """EpiKV score of every position 0..T-1 of one sequence.
 
@@ -116,6 +140,41 @@ def lag_token_variance(k_t, v_t, k_prev_chunk, v_prev_chunk, eps=LAG_EPS):
         var = ((xn - mu) ** 2).mean(axis=-1)              # over head dim, [L, H]
         total = var if total is None else total + var     # key + value
     return float(total.mean())                            # over (layer, head)
+
+
+def head_variance(x):
+    """mean over (layer, head) of the population variance over the head
+    dimension of one token's stored vectors x [L, H, d] (Sec. 3.3, KV-key /
+    KV-val, reading R12)."""
+    x = np.asarray(x, dtype=np.float64)
+    mu = x.mean(axis=-1, keepdims=True)
+    return float(((x - mu) ** 2).mean(axis=-1).mean())
+
+
+def kv_variance_scores(X, w=64):
+    """KV-key (X = keys) or KV-val (X = values) scores: the rolling mean of
+    the per-token head variance (Sec. 3.3, Tab. 1, R12)."""
+    return rolling_mean(np.array([head_variance(X[t]) for t in range(X.shape[0])]), w)
+
+
+def lag_key_token_variance(k_t, k_prev_chunk, eps=LAG_EPS):
+    """The key term of Lag-KV for one token (reading R13)."""
+    x = np.asarray(k_t, dtype=np.float64)
+    prev = np.asarray(k_prev_chunk, dtype=np.float64)
+    mn = prev.min(axis=0)
+    mx = prev.max(axis=0)
+    xn = (x - mn) / (mx - mn + eps)
+    return float(((xn - xn.mean(axis=-1, keepdims=True)) ** 2).mean(axis=-1).mean())
+
+
+def lag_key_scores(K, lag=16, eps=LAG_EPS, w=64):
+    """lag-kv-key scores: rolling mean of the key-only Lag-KV term (R13)."""
+    T = K.shape[0]
+    u = np.zeros(T)
+    for t in range(lag, T):
+        c = t // lag
+        u[t] = lag_key_token_variance(K[t], K[(c - 1) * lag: c * lag], eps)
+    return rolling_mean(u, w)
 
 
 def lag_variance_trace(K, V, lag=16, eps=LAG_EPS):

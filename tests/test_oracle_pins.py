@@ -331,3 +331,54 @@ def test_simulate_decode_keeps_structure():
         assert after[-64:] == before[-64:]                   # R = min(128, 64)
         assert after == sorted(after)
     assert len(final) <= 256 + 15
+
+
+# ------------------------------------------- the other attention-free variants
+def test_hsvar_closed_forms():
+    # a walk with constant step a in Band A and b in Band B: g-bar = a, b
+    T, D = 150, 8
+    ra = np.zeros((T, D)); ra[:, 0] = 3.0 * np.arange(T)
+    rb = np.zeros((T, D)); rb[:, 1] = 0.5 * np.arange(T)
+    s = O.hsvar_scores([ra], [rb], w=16)
+    assert s[0] == 0.0
+    np.testing.assert_allclose(s[1:], 2.5, rtol=1e-14)
+    # linear drift with a full window: mean = a + b (t - (w - 1) / 2)
+    t = np.arange(300, dtype=np.float64)
+    g = 2.0 + 0.25 * t
+    m = O.rolling_band_mean(g, 64)
+    np.testing.assert_allclose(m[70:], 2.0 + 0.25 * (t[70:] - 31.5), rtol=1e-13)
+    # warm-up averages positions 1..t only, never position 0
+    g2 = np.array([1e9, 1.0, 2.0, 6.0])
+    np.testing.assert_allclose(O.rolling_band_mean(g2, 64), [0.0, 1.0, 1.5, 3.0])
+    # swapping the bands negates the score
+    rng = np.random.default_rng(15)
+    A, B = rng.normal(size=(2, 90, 12))
+    np.testing.assert_allclose(O.hsvar_scores([B], [A], 8), -O.hsvar_scores([A], [B], 8), rtol=1e-13)
+
+
+def test_head_variance_closed_forms_and_equivariance():
+    x = np.zeros((1, 1, 8))
+    x[0, 0, 3] = 4.0                             # one-hot: var = a^2 (d - 1) / d^2
+    assert O.head_variance(x) == pytest.approx(16.0 * 7 / 64, rel=1e-15)
+    assert O.head_variance(np.full((2, 3, 16), 7.5)) == 0.0
+    rng = np.random.default_rng(16)
+    X = rng.normal(size=(2, 3, 16))
+    v = O.head_variance(X)
+    assert O.head_variance(-2.0 * X + 100.0) == pytest.approx(4.0 * v, rel=1e-12)
+    # mean over (layer, head), not a sum: a duplicated head keeps it
+    assert O.head_variance(np.concatenate([X, X], axis=1)) == pytest.approx(v, rel=1e-14)
+    s = O.kv_variance_scores(np.stack([X, 2 * X, 3 * X]), w=64)
+    np.testing.assert_allclose(s, [v, 2.5 * v, 14.0 / 3.0 * v], rtol=1e-12)
+
+
+def test_lag_key_is_the_key_half_of_lagkv():
+    K, V, u, _ = _golden_lag()
+    # the hand example's V terms vanish at t = 2, 3 and equal 1/4 at t = 4
+    uk = [O.lag_key_token_variance(K[t], K[(t // 2 - 1) * 2:(t // 2) * 2], 1e-300) for t in (2, 3, 4)]
+    np.testing.assert_allclose(uk, [1 / 64, 1 / 4, 1 / 4], rtol=1e-14)
+    rng = np.random.default_rng(17)
+    K = rng.normal(size=(64, 2, 2, 8))
+    V = rng.normal(size=(64, 2, 2, 8))
+    both = O.lagkv_scores(K, V, lag=8)
+    np.testing.assert_allclose(O.lag_key_scores(K, lag=8) + O.lag_key_scores(V, lag=8), both, rtol=1e-12)
+    np.testing.assert_array_equal(O.lag_key_scores(K, lag=8)[:8], 0.0)
