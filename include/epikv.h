@@ -62,8 +62,22 @@ typedef enum {
   EPIKV_DEV_TIMEOUT = 6,    /* a bounded wait inside a kernel gave up */
 } epikv_device_error;
 
-/* Score kinds (bit mask in epikv_config.score_kinds, one value as policy). */
-enum { EPIKV_SCORE_BANDZ = 1, EPIKV_SCORE_LAGKV = 2 };
+/* Score kinds (bit mask in epikv_config.score_kinds, one value as policy).
+ *   BANDZ   EpiKV: Band A mean - Band B mean of rolling z-scores of g (Eq. 3)
+ *   LAGKV   Lag-KV: lag-normalised key + value head variance (Sec. 3.3)
+ *   HSVAR   HS-variance: Band A mean - Band B mean of rolling means of g (Eq. 2)
+ *   KVKEY   KV-key: rolling mean of the stored keys' head variance (Sec. 3.3)
+ *   KVVAL   KV-val: the same for the values (Sec. 3.3)
+ *   LAGKEY  lag-kv-key: Lag-KV's key term only (Tab. "acc-math" rows)
+ * The band kinds use z_window as their window; the K/V kinds lag_window. */
+enum {
+  EPIKV_SCORE_BANDZ = 1,
+  EPIKV_SCORE_LAGKV = 2,
+  EPIKV_SCORE_HSVAR = 4,
+  EPIKV_SCORE_KVKEY = 8,
+  EPIKV_SCORE_KVVAL = 16,
+  EPIKV_SCORE_LAGKEY = 32,
+};
 
 /* KV cache layouts. */
 enum { EPIKV_LAYOUT_CONTIGUOUS = 0, EPIKV_LAYOUT_PAGED = 1 };
@@ -78,13 +92,13 @@ typedef struct {
   int32_t hidden;           /* D: hidden size, a multiple of 8, <= 8192 */
   int32_t n_band_a;         /* Band A layers passed per update (Sec. 3.2: 7..13) */
   int32_t n_band_b;         /* Band B layers (Sec. 3.2: 18..25); A+B <= 32 */
-  int32_t z_window;         /* w of Eq. 3 (paper: 64), 1..1024 */
+  int32_t z_window;         /* w of Eq. 2 and 3 (paper: 64), 1..1024 */
   float z_eps;              /* epsilon of Eq. 3 (1e-6) */
   int32_t lag;              /* Lag-KV chunk length (16), >= 1 */
   float lag_eps;            /* epsilon of the range normalisation (1e-6) */
-  int32_t lag_window;       /* rolling-mean window of the Lag-KV score (64), 1..1024 */
+  int32_t lag_window;       /* rolling-mean window of the K/V scores (64), 1..1024 */
   int32_t recency_cap;      /* recency window R = min(recency_cap, K/4) (App. D: 128) */
-  int32_t score_kinds;      /* EPIKV_SCORE_* mask computed by every update */
+  int32_t score_kinds;      /* EPIKV_SCORE_* mask (1..63) computed by every update */
 } epikv_config;
 
 /* New hidden-state rows of one update call (Sec. 3.1: the per-layer hidden
@@ -147,9 +161,10 @@ epikv_status epikv_seq_reset(epikv_ctx* ctx, int32_t seq, int32_t prefill_len, i
  *                       (d_cu_new[0] = 0, non-decreasing)
  *   max_new             host: an upper bound of every entry's new tokens
  *                       (<= cfg.max_new_tokens; sizes the grid)
- *   hidden              band rows of the new tokens (needed for BANDZ)
+ *   hidden              band rows of the new tokens (needed for BANDZ, HSVAR)
  *   kv                  the cache; the new tokens' K/V rows must already be
- *                       in slots n_cache .. n_cache+n_new-1 (needed for LAGKV)
+ *                       in slots n_cache .. n_cache+n_new-1 (needed for the
+ *                       K/V kinds)
  * Each token's score is computed once, causally, and frozen (Sec. 3.3). */
 epikv_status epikv_score_update(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
                                 const int32_t* d_cu_new, int32_t max_new,

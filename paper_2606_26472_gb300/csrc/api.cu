@@ -40,17 +40,17 @@ bool valid_config(const epikv_config* c) {
   if (c->max_seqs < 1 || c->max_seqs > 4096) return false;
   if (c->max_cache_tokens < 1 || c->max_cache_tokens > (1 << 24)) return false;
   if (c->max_new_tokens < 1 || c->max_new_tokens > (1 << 20)) return false;
-  if (c->score_kinds < 1 || c->score_kinds > 3) return false;
+  if (c->score_kinds < 1 || c->score_kinds > 63) return false;
   if (c->recency_cap < 0) return false;
   if (c->num_layers < 1 || c->num_kv_heads < 1 || c->num_kv_heads > 32) return false;
   if (!is_pow2(c->head_dim) || c->head_dim < 8 || c->head_dim > 256) return false;
   if (c->num_kv_heads * c->head_dim / 8 > 256) return false;
-  if (c->score_kinds & EPIKV_SCORE_BANDZ) {
+  if (c->score_kinds & kBandKinds) {
     if (c->hidden < 8 || c->hidden % 8 != 0 || c->hidden > 8192) return false;
     if (c->n_band_a < 1 || c->n_band_b < 1 || c->n_band_a + c->n_band_b > kMaxBand) return false;
     if (c->z_window < 1 || c->z_window > 1024 || !(c->z_eps >= 0.f)) return false;
   }
-  if (c->score_kinds & EPIKV_SCORE_LAGKV) {
+  if (c->score_kinds & kKvKinds) {
     if (c->lag < 1 || c->lag_window < 1 || c->lag_window > 1024 || !(c->lag_eps >= 0.f)) return false;
     if ((int64_t)c->max_new_tokens * 2 * c->num_layers > (int64_t)1 << 30) return false;
   }
@@ -68,7 +68,7 @@ Dims make_dims(const epikv_config* c) {
   d.d = c->head_dim;
   d.kinds = c->score_kinds;
   d.recency_cap = c->recency_cap;
-  const bool bz = c->score_kinds & EPIKV_SCORE_BANDZ, lg = c->score_kinds & EPIKV_SCORE_LAGKV;
+  const bool bz = c->score_kinds & kBandKinds, lg = c->score_kinds & kKvKinds;
   d.D = bz ? c->hidden : 0;
   d.nA = bz ? c->n_band_a : 0;
   d.nB = bz ? c->n_band_b : 0;
@@ -105,18 +105,20 @@ size_t carve(const Dims& d, DevState* st, char* base) {
   st->pos = (int32_t*)take(S * T * 4);
   st->kept = (int32_t*)take(S * T * 4);
   st->n_kept = (int32_t*)take(S * 4);
-  if (d.kinds & EPIKV_SCORE_BANDZ) {
+  for (int k = 0; k < kNumKinds; ++k)
+    if (d.kinds & (1 << k)) st->score[k] = (float*)take(S * T * 4);
+  if (d.kinds & kBandKinds) {
     const size_t nb = d.nA + d.nB;
-    st->score[0] = (float*)take(S * T * 4);
     st->h_prev = (__nv_bfloat16*)take(S * 2 * nb * d.D * 2);
     st->g_ring = (float*)take(S * nb * d.G * 4);
   }
-  if (d.kinds & EPIKV_SCORE_LAGKV) {
-    st->score[1] = (float*)take(S * T * 4);
+  if (d.kinds & kNormKinds) {
     st->lag_rng = (__nv_bfloat16*)take(S * d.L * 2 * 4 * (size_t)d.H * d.d * 2);
     st->lag_part = (float*)take(S * (size_t)d.max_new * 2 * d.L * 4);
-    st->u_ring = (float*)take(S * (size_t)d.G * 4);
   }
+  if (d.kinds & kRawKinds) st->raw_part = (float*)take(S * (size_t)d.max_new * 2 * d.L * 4);
+  for (int q = 0; q < 4; ++q)
+    if (d.kinds & kv_kind(q)) st->u_ring[q] = (float*)take(S * (size_t)d.G * 4);
   return align_up(off, 256);
 }
 
@@ -149,7 +151,7 @@ bool valid_kv(const epikv_ctx* ctx, const epikv_kv_view* kv, KvDev* out) {
 }
 
 bool valid_hidden(const epikv_ctx* ctx, const epikv_hidden_view* hv) {
-  if (!(ctx->dm.kinds & EPIKV_SCORE_BANDZ)) return true;
+  if (!(ctx->dm.kinds & kBandKinds)) return true;
   if (!hv || hv->row_stride < ctx->dm.D || hv->row_stride % 8) return false;
   for (int i = 0; i < ctx->dm.nA + ctx->dm.nB; ++i)
     if (!hv->band_rows[i] || !aligned16(hv->band_rows[i])) return false;
@@ -201,8 +203,7 @@ epikv_status epikv_init(epikv_ctx** out, const epikv_config* cfg, void* d_worksp
 epikv_status epikv_seq_reset(epikv_ctx* ctx, int32_t seq, int32_t prefill_len, int32_t policy,
                              cudaStream_t stream) {
   if (!ctx || seq < 0 || seq >= ctx->dm.S || prefill_len < 0) return EPIKV_EINVAL;
-  if ((policy != EPIKV_SCORE_BANDZ && policy != EPIKV_SCORE_LAGKV) || !(policy & ctx->dm.kinds))
-    return EPIKV_EINVAL;
+  if (policy < 1 || (policy & (policy - 1)) || !(policy & ctx->dm.kinds)) return EPIKV_EINVAL;
   ctx->last_stream = stream;
   return cuda_status(launch_reset_seq(ctx->st, ctx->dm, seq, prefill_len, policy, stream));
 }
@@ -216,7 +217,7 @@ static epikv_status score_update_impl(epikv_ctx* ctx, int32_t n_seq, const int32
   if (!valid_hidden(ctx, hidden)) return EPIKV_EINVAL;
   KvDev kd;
   memset(&kd, 0, sizeof(kd));
-  if ((ctx->dm.kinds & EPIKV_SCORE_LAGKV) && !valid_kv(ctx, kv, &kd)) return EPIKV_EINVAL;
+  if ((ctx->dm.kinds & kKvKinds) && !valid_kv(ctx, kv, &kd)) return EPIKV_EINVAL;
   ctx->last_stream = stream;
   return cuda_status(launch_score_update(ctx->st, ctx->dm, n_seq, d_seq_ids, d_cu_new, max_new, hidden, &kd,
                                          ctx->num_sms, stream, launches));
@@ -295,7 +296,7 @@ epikv_status epikv_set_phase_events(epikv_ctx* ctx, const cudaEvent_t* events) {
 epikv_status epikv_read_slots(epikv_ctx* ctx, int32_t seq, int32_t kind, float* h_score, int32_t* h_pos,
                               int32_t cap, int32_t* h_n) {
   if (!ctx || seq < 0 || seq >= ctx->dm.S || cap < 0 || !h_n) return EPIKV_EINVAL;
-  if (h_score && (kind < 1 || kind > 2 || !(kind & ctx->dm.kinds))) return EPIKV_EINVAL;
+  if (h_score && (kind < 1 || (kind & (kind - 1)) || !(kind & ctx->dm.kinds))) return EPIKV_EINVAL;
   cudaError_t e = cudaStreamSynchronize(ctx->last_stream);
   int32_t n = 0;
   if (e == cudaSuccess) e = cudaMemcpy(&n, ctx->st.n_cache + seq, 4, cudaMemcpyDeviceToHost);
@@ -305,7 +306,7 @@ epikv_status epikv_read_slots(epikv_ctx* ctx, int32_t seq, int32_t kind, float* 
   if (m > 0 && h_pos)
     e = cudaMemcpy(h_pos, ctx->st.pos + (size_t)seq * ctx->dm.T, (size_t)m * 4, cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && m > 0 && h_score)
-    e = cudaMemcpy(h_score, ctx->st.score[kind - 1] + (size_t)seq * ctx->dm.T, (size_t)m * 4,
+    e = cudaMemcpy(h_score, ctx->st.score[kind_index(kind)] + (size_t)seq * ctx->dm.T, (size_t)m * 4,
                    cudaMemcpyDeviceToHost);
   return cuda_status(e);
 }

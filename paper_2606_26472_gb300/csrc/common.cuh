@@ -13,6 +13,24 @@
 namespace epikv {
 
 constexpr int kMaxBand = 32;
+constexpr int kNumKinds = 6;  // score kind index k <-> mask bit (1 << k)
+constexpr int kBandKinds = EPIKV_SCORE_BANDZ | EPIKV_SCORE_HSVAR;
+constexpr int kNormKinds = EPIKV_SCORE_LAGKV | EPIKV_SCORE_LAGKEY;   // need the chunk ranges
+constexpr int kRawKinds = EPIKV_SCORE_KVKEY | EPIKV_SCORE_KVVAL;
+constexpr int kKvKinds = kNormKinds | kRawKinds;
+// the K/V kinds in the order of their rolling-mean rings
+__host__ __device__ __forceinline__ int kv_kind(int q) {
+  return q == 0 ? EPIKV_SCORE_LAGKV : q == 1 ? EPIKV_SCORE_KVKEY : q == 2 ? EPIKV_SCORE_KVVAL : EPIKV_SCORE_LAGKEY;
+}
+
+__host__ __device__ __forceinline__ int kind_index(int bit) {
+  int k = 0;
+  while (bit > 1) {
+    bit >>= 1;
+    ++k;
+  }
+  return k;
+}
 
 // Device pointers carved out of the caller's workspace (one context).
 struct DevState {
@@ -25,13 +43,14 @@ struct DevState {
   uint32_t* ticket;        // [S] last-CTA tickets of the finalize kernel
   int32_t* err;            // [1] sticky device error word
   unsigned long long* stats;  // [4] epikv_stats
-  float* score[2];         // [S][T] frozen scores (kind 0 = band-z, 1 = Lag-KV)
+  float* score[kNumKinds]; // [S][T] frozen scores per kind (null when the kind is off)
   int32_t* pos;            // [S][T] position of each slot
   __nv_bfloat16* h_prev;   // [S][2][n_band][D] last hidden row per band layer
   float* g_ring;           // [S][n_band][G] g by position (mod G)
   __nv_bfloat16* lag_rng;  // [S][L][2][4][H][d] prev min, prev max, cur min, cur max
-  float* lag_part;         // [S][max_new][2L] per-(layer, K|V) head-summed variances
-  float* u_ring;           // [S][G] u by position (mod G)
+  float* lag_part;         // [S][max_new][2L] per-(layer, K|V) head-summed normalised variances
+  float* raw_part;         // [S][max_new][2L] per-(layer, K|V) head-summed raw variances
+  float* u_ring[4];        // [S][G] per K/V kind (kv_kind order): u by position (mod G)
   int32_t* kept;           // [S][T] kept lists of epikv_step
   int32_t* n_kept;         // [S]
 };

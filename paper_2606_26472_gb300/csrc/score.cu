@@ -224,10 +224,12 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
     return;
   }
   const int ch = h * dm.d + q * 8;  // first channel of this thread within the token row
-  __nv_bfloat16* rng = st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd;
+  const bool need_norm = dm.kinds & kNormKinds;   // uniform across the grid
+  const bool need_raw = dm.kinds & kRawKinds;
+  __nv_bfloat16* rng = need_norm ? st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd : nullptr;
 
   uint4 pmn = make_uint4(0, 0, 0, 0), pmx = pmn, cmn = pmn, cmx = pmn;
-  if (active) {
+  if (active && need_norm) {
     pmn = *reinterpret_cast<const uint4*>(rng + 0 * hd + ch);
     pmx = *reinterpret_cast<const uint4*>(rng + 1 * hd + ch);
     cmn = *reinterpret_cast<const uint4*>(rng + 2 * hd + ch);
@@ -240,7 +242,9 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
   const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
   __shared__ int64_t soff[kLagOffs];
   __shared__ float hv[2][kLagSeg][32];  // [segment parity][token][head]; the host admits H <= 32
-  float* part = st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L);
+  __shared__ float hr[2][kLagSeg][32];  // raw variances, same layout
+  float* part = need_norm ? st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
+  float* rpart = need_raw ? st.raw_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
   int r = p0 % dm.lag;                   // position of the next token inside its chunk
   int parity = 0;
 
@@ -267,8 +271,23 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
 #pragma unroll
       for (int j = 0; j < kLagSeg; ++j) {
         if (j < seg) {
+          if (need_raw) {  // population variance of the stored vector over the head dimension
+            float xf[8], s1 = 0.f;
+            unpack8(x[j], xf);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s1 += xf[e];
+            const float mean = group_sum(s1, LH) * inv_d;
+            float s2 = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float dv = xf[e] - mean;
+              s2 = fmaf(dv, dv, s2);
+            }
+            const float var_raw = group_sum(s2, LH) * inv_d;
+            if (q == 0 && active) hr[parity][j][h] = var_raw;
+          }
           float var = 0.f;
-          if (has_prev) {  // uniform across the block
+          if (has_prev && need_norm) {  // uniform across the block
             float xf[8], s1 = 0.f, s2 = 0.f;
             unpack8(x[j], xf);
 #pragma unroll
@@ -301,9 +320,16 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
         }
       __syncthreads();
       if (tid < seg) {
-        float sum = 0.f;
-        for (int hh = 0; hh < dm.H; ++hh) sum += hv[parity][tid][hh];
-        part[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+        if (need_norm) {
+          float sum = 0.f;
+          for (int hh = 0; hh < dm.H; ++hh) sum += hv[parity][tid][hh];
+          part[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+        }
+        if (need_raw) {
+          float sum = 0.f;
+          for (int hh = 0; hh < dm.H; ++hh) sum += hr[parity][tid][hh];
+          rpart[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+        }
       }
       parity ^= 1;
       r += seg;
@@ -316,7 +342,7 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
       i += seg;
     }
   }
-  if (active) {
+  if (active && need_norm) {
     *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = pmn;
     *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = pmx;
     *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = cmn;
@@ -356,7 +382,7 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
       const int pos = p0 + i;
       if (lane == 0) st.pos[(size_t)seq * dm.T + nc0 + i] = pos;
     }
-    if (dm.kinds & EPIKV_SCORE_BANDZ) {
+    if (dm.kinds & kBandKinds) {
       // every g value the tile's windows reach, all band layers, one round of loads
       extern __shared__ float sg[];  // [nb][span]
       const int span = kFinTile + dm.z_window - 1;
@@ -375,63 +401,88 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
         const int i = i0 + sub;
         const int pos = p0 + i;
         const bool live = i < i_hi && pos >= 1 && band < nb;
-        float za = 0.f, zb = 0.f;
+        float za = 0.f, zb = 0.f, ma = 0.f, mb = 0.f;
         if (live) {
           const int n = min(dm.z_window, pos);
           const float* row = sg + band * span + (pos - pos_base);   // row[-k] = g at position pos - k
-          const float gnew = row[0];
-          float dsum = 0.f;
-          for (int k = 0; k < n; ++k) dsum += row[-k] - gnew;
-          const float mean_d = dsum / (float)n;
-          float dev = 0.f;
-          for (int k = 0; k < n; ++k) {
-            const float e = (row[-k] - gnew) - mean_d;
-            dev = fmaf(e, e, dev);
+          if (dm.kinds & EPIKV_SCORE_BANDZ) {
+            const float gnew = row[0];
+            float dsum = 0.f;
+            for (int k = 0; k < n; ++k) dsum += row[-k] - gnew;
+            const float mean_d = dsum / (float)n;
+            float dev = 0.f;
+            for (int k = 0; k < n; ++k) {
+              const float e = (row[-k] - gnew) - mean_d;
+              dev = fmaf(e, e, dev);
+            }
+            const float sigma = sqrtf(dev / (float)n);
+            const float z = -mean_d / (sigma + dm.z_eps);  // g(t) - mu = -(mean of g - g(t))
+            if (band < dm.nA) za = z; else zb = z;
           }
-          const float sigma = sqrtf(dev / (float)n);
-          const float z = -mean_d / (sigma + dm.z_eps);  // g(t) - mu = -(mean of g - g(t))
-          if (band < dm.nA) za = z; else zb = z;
+          if (dm.kinds & EPIKV_SCORE_HSVAR) {  // rolling mean of g (Eq. 2)
+            float sum = 0.f;
+            for (int k = 0; k < n; ++k) sum += row[-k];
+            const float gbar = sum / (float)n;
+            if (band < dm.nA) ma = gbar; else mb = gbar;
+          }
         }
         for (int o = lpt >> 1; o > 0; o >>= 1) {  // stays inside each token's lane group
           za += __shfl_xor_sync(0xffffffffu, za, o);
           zb += __shfl_xor_sync(0xffffffffu, zb, o);
+          ma += __shfl_xor_sync(0xffffffffu, ma, o);
+          mb += __shfl_xor_sync(0xffffffffu, mb, o);
         }
-        if (band == 0 && i < i_hi)
-          st.score[0][(size_t)seq * dm.T + nc0 + i] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
+        if (band == 0 && i < i_hi) {
+          const size_t slot = (size_t)seq * dm.T + nc0 + i;
+          if (dm.kinds & EPIKV_SCORE_BANDZ)
+            st.score[0][slot] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
+          if (dm.kinds & EPIKV_SCORE_HSVAR)
+            st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
+        }
       }
     }
-    if (dm.kinds & EPIKV_SCORE_LAGKV) {
+    if (dm.kinds & kKvKinds) {
       __shared__ float su[kFinTile + kMaxWindow];
       const int w = dm.lag_window;
       const int lo = max(0, i_lo - (w - 1));
-      const float* part = st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L);
       const float inv_lh = 1.f / (float)(dm.L * dm.H);
-      for (int i = lo + tid; i < i_hi; i += kFinThreads) {
-        const int pos = p0 + i;
-        float u = 0.f;
-        if (pos >= dm.lag) {
-          const float* pp = part + (size_t)i * (2 * dm.L);
-          float s = 0.f;
-          for (int q = 0; q < 2 * dm.L; ++q) s += pp[q];
-          u = s * inv_lh;
+      for (int qk = 0; qk < 4; ++qk) {
+        const int kind = kv_kind(qk);
+        if (!(dm.kinds & kind)) continue;
+        // which partials: normalised or raw; all (layer, K|V) entries, keys only or values only
+        const bool raw = kind & kRawKinds;
+        const float* part = (raw ? st.raw_part : st.lag_part) + (size_t)seq * dm.max_new * (2 * dm.L);
+        const int q0 = kind == EPIKV_SCORE_KVVAL ? 1 : 0;
+        const int qs = kind == EPIKV_SCORE_LAGKV ? 1 : 2;
+        float* ring = st.u_ring[qk] + (size_t)seq * dm.G;
+        float* out = st.score[kind_index(kind)] + (size_t)seq * dm.T + nc0;
+        __syncthreads();  // su is reused kind after kind
+        for (int i = lo + tid; i < i_hi; i += kFinThreads) {
+          const int pos = p0 + i;
+          float u = 0.f;
+          if (raw || pos >= dm.lag) {  // the normalised kinds have no value in chunk 0
+            const float* pp = part + (size_t)i * (2 * dm.L);
+            float s = 0.f;
+            for (int q = q0; q < 2 * dm.L; q += qs) s += pp[q];
+            u = s * inv_lh;
+          }
+          su[i - lo] = u;
         }
-        su[i - lo] = u;
-      }
-      __syncthreads();
-      for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
-        const int pos = p0 + i;
-        const int n = min(w, pos + 1);
-        float acc = 0.f;
+        __syncthreads();
+        for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
+          const int pos = p0 + i;
+          const int n = min(w, pos + 1);
+          float acc = 0.f;
 #pragma unroll
-        for (int m = 0; m < WPL; ++m) {
-          const int k = lane + 32 * m;
-          if (k < n) acc += (i - k >= 0) ? su[i - k - lo] : st.u_ring[(size_t)seq * dm.G + ((pos - k) & Gm)];
+          for (int m = 0; m < WPL; ++m) {
+            const int k = lane + 32 * m;
+            if (k < n) acc += (i - k >= 0) ? su[i - k - lo] : ring[(pos - k) & Gm];
+          }
+          const float mean = warp_sum(acc) / (float)n;
+          if (lane == 0) out[i] = mean;
         }
-        const float mean = warp_sum(acc) / (float)n;
-        if (lane == 0) st.score[1][(size_t)seq * dm.T + nc0 + i] = mean;
+        for (int i = i_lo + tid; i < i_hi; i += kFinThreads) ring[(p0 + i) & Gm] = su[i - lo];
       }
-      for (int i = i_lo + tid; i < i_hi; i += kFinThreads)
-        st.u_ring[(size_t)seq * dm.G + ((p0 + i) & Gm)] = su[i - lo];
     }
   }
 
@@ -445,7 +496,7 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
       if (fits) {
         st.n_cache[seq] = nc0 + n_new;
         st.n_seen[seq] = p0 + n_new;
-        if ((dm.kinds & EPIKV_SCORE_BANDZ) && n_new > 0) st.hp_parity[seq] ^= 1;
+        if ((dm.kinds & kBandKinds) && n_new > 0) st.hp_parity[seq] ^= 1;
         atomicAdd(&st.stats[0], (unsigned long long)n_new);
       }
       st.ticket[seq] = 0u;
@@ -456,7 +507,7 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
 // ------------------------------------------------------------------ launchers
 // dynamic shared memory of the finalize kernel: the band windows of a tile
 static size_t finalize_smem(const Dims& dm) {
-  if (!(dm.kinds & EPIKV_SCORE_BANDZ)) return 0;
+  if (!(dm.kinds & kBandKinds)) return 0;
   return (size_t)(dm.nA + dm.nB) * (kFinTile + dm.z_window - 1) * sizeof(float);
 }
 
@@ -474,7 +525,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
                                 const KvDev* kv, int num_sms, cudaStream_t stream, int* launches) {
   if (n_seq == 0 || max_new == 0) return cudaSuccess;
   const int nb = dm.nA + dm.nB;
-  if (dm.kinds & EPIKV_SCORE_BANDZ) {
+  if (dm.kinds & kBandKinds) {
     BandRows rows;
     for (int i = 0; i < kMaxBand; ++i)
       rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
@@ -499,7 +550,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
       bandz_g_kernel<4><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
     ++*launches;
   }
-  if (dm.kinds & EPIKV_SCORE_LAGKV) {
+  if (dm.kinds & kKvKinds) {
     dim3 grid(2 * dm.L, n_seq);
     const int threads = max(32, (dm.H * dm.d / 8 + 31) / 32 * 32);
     switch (dm.d / 8) {
@@ -514,8 +565,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
   }
   {
     dim3 grid((max_new + kFinTile - 1) / kFinTile, n_seq);
-    const int wmax = max((dm.kinds & EPIKV_SCORE_BANDZ) ? dm.z_window : 1,
-                         (dm.kinds & EPIKV_SCORE_LAGKV) ? dm.lag_window : 1);
+    const int wmax = max((dm.kinds & kBandKinds) ? dm.z_window : 1, (dm.kinds & kKvKinds) ? dm.lag_window : 1);
     const int wpl = (wmax + 31) / 32;
     const size_t smem = finalize_smem(dm);
     if (wpl <= 1)

@@ -110,8 +110,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
     }
     return;
   }
-  const int kind = st.policy[seq] == EPIKV_SCORE_LAGKV ? 1 : 0;
-  const float* __restrict__ sc = st.score[kind] + (size_t)seq * dm.T;
+  const float* __restrict__ sc = st.score[kind_index(st.policy[seq])] + (size_t)seq * dm.T;
   int32_t* out = kept_out + (size_t)b * kept_stride;
 
   __shared__ uint32_t hist[256];
@@ -204,23 +203,22 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   __syncthreads();  // kept list visible to the whole block
 
   // ---- compact slot metadata in place (kept[i] >= i, increasing i)
-  float* s0 = st.score[0] ? st.score[0] + (size_t)seq * dm.T : nullptr;
-  float* s1 = st.score[1] ? st.score[1] + (size_t)seq * dm.T : nullptr;
   int32_t* ps = st.pos + (size_t)seq * dm.T;
   for (int j0 = fe; j0 < n_kept; j0 += kSelThreads) {
     const int j = j0 + tid;
-    float v0 = 0.f, v1 = 0.f;
+    float v[kNumKinds];
     int32_t p = 0;
     if (j < n_kept) {
       const int src = out[j];
-      if (s0) v0 = s0[src];
-      if (s1) v1 = s1[src];
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k) v[k] = st.score[k] ? st.score[k][(size_t)seq * dm.T + src] : 0.f;
       p = ps[src];
     }
     __syncthreads();
     if (j < n_kept) {
-      if (s0) s0[j] = v0;
-      if (s1) s1[j] = v1;
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k)
+        if (st.score[k]) st.score[k][(size_t)seq * dm.T + j] = v[k];
       ps[j] = p;
     }
     __syncthreads();

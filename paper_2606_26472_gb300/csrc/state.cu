@@ -5,7 +5,7 @@
 namespace epikv {
 
 __global__ void init_state_kernel(DevState st, Dims dm) {
-  const int default_policy = (dm.kinds & EPIKV_SCORE_BANDZ) ? EPIKV_SCORE_BANDZ : EPIKV_SCORE_LAGKV;
+  const int default_policy = dm.kinds & -dm.kinds;  // the lowest enabled kind
   for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < dm.S; s += gridDim.x * blockDim.x)
     st.policy[s] = default_policy;
 }

@@ -13,7 +13,8 @@ LIB_PATH = os.path.join(_HERE, "libepikv.so")
 EPIKV_OK, EPIKV_EINVAL, EPIKV_ECUDA, EPIKV_EDEVICE = 0, 1, 2, 3
 EPIKV_DEV_OK, EPIKV_DEV_BATCH, EPIKV_DEV_CAPACITY, EPIKV_DEV_SLOT = 0, 1, 2, 3
 EPIKV_DEV_KEPT, EPIKV_DEV_BUDGET, EPIKV_DEV_TIMEOUT = 4, 5, 6
-EPIKV_SCORE_BANDZ, EPIKV_SCORE_LAGKV = 1, 2
+EPIKV_SCORE_BANDZ, EPIKV_SCORE_LAGKV, EPIKV_SCORE_HSVAR = 1, 2, 4
+EPIKV_SCORE_KVKEY, EPIKV_SCORE_KVVAL, EPIKV_SCORE_LAGKEY = 8, 16, 32
 EPIKV_LAYOUT_CONTIGUOUS, EPIKV_LAYOUT_PAGED = 0, 1
 
 

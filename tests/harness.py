@@ -21,7 +21,10 @@ from synth import gen
 from synth.device import DeviceTrace, as_u16
 
 TOL = 1e-4
-KIND_INDEX = {E.EPIKV_SCORE_BANDZ: 0, E.EPIKV_SCORE_LAGKV: 1}
+ALL_KINDS = (E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV, E.EPIKV_SCORE_HSVAR, E.EPIKV_SCORE_KVKEY,
+             E.EPIKV_SCORE_KVVAL, E.EPIKV_SCORE_LAGKEY)
+BAND_KINDS = E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR
+KV_KINDS = E.EPIKV_SCORE_LAGKV | E.EPIKV_SCORE_KVKEY | E.EPIKV_SCORE_KVVAL | E.EPIKV_SCORE_LAGKEY
 
 
 def assert_scores_close(gpu, ref, what=""):
@@ -41,16 +44,26 @@ class OracleTrace:
         self.length = length
         pos = np.arange(length)
         self.scores = {}
-        if kinds & E.EPIKV_SCORE_BANDZ:
+        if kinds & (E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR):
             seg = gen.segment_index(model, seq, length)
             ra = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_a]
             rb = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_b]
-            self.scores[E.EPIKV_SCORE_BANDZ] = O.bandz_scores(ra, rb, z_window)
-        if kinds & E.EPIKV_SCORE_LAGKV:
+            if kinds & E.EPIKV_SCORE_BANDZ:
+                self.scores[E.EPIKV_SCORE_BANDZ] = O.bandz_scores(ra, rb, z_window)
+            if kinds & E.EPIKV_SCORE_HSVAR:
+                self.scores[E.EPIKV_SCORE_HSVAR] = O.hsvar_scores(ra, rb, z_window)
+        if kinds & KV_KINDS:
             sp = gen.spike_flags(model, seq, length)
             K = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0, pos, sp))
             V = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 1, pos, sp))
-            self.scores[E.EPIKV_SCORE_LAGKV] = O.lagkv_scores(K, V, lag, w=lag_window)
+            if kinds & E.EPIKV_SCORE_LAGKV:
+                self.scores[E.EPIKV_SCORE_LAGKV] = O.lagkv_scores(K, V, lag, w=lag_window)
+            if kinds & E.EPIKV_SCORE_LAGKEY:
+                self.scores[E.EPIKV_SCORE_LAGKEY] = O.lag_key_scores(K, lag, w=lag_window)
+            if kinds & E.EPIKV_SCORE_KVKEY:
+                self.scores[E.EPIKV_SCORE_KVKEY] = O.kv_variance_scores(K, lag_window)
+            if kinds & E.EPIKV_SCORE_KVVAL:
+                self.scores[E.EPIKV_SCORE_KVVAL] = O.kv_variance_scores(V, lag_window)
 
 
 class Session:
@@ -92,7 +105,7 @@ class Session:
         self.kv = self.cache.view()
         nb = len(model.band_a) + len(model.band_b)
         self.hid = torch.empty((nb, n_seq * max_new, model.hidden), dtype=torch.bfloat16, device=device) \
-            if kinds & E.EPIKV_SCORE_BANDZ else None
+            if kinds & BAND_KINDS else None
         self.n_cache = [0] * n_seq
         self.n_seen = [0] * n_seq
         self.kept = torch.empty((n_seq, max_tokens), dtype=torch.int32, device=device)
@@ -212,7 +225,41 @@ def oracle_bandz_at(model, tabs, seq, t, w=64):
     return float(O.epiphany_score([z[l] for l in model.band_a], [z[l] for l in model.band_b])[0])
 
 
-def oracle_lag_at(model, tabs, seq, t, lag=16, w=64):
+def oracle_hsvar_at(model, tabs, seq, t, w=64):
+    """fp64 HS-variance score of position t from the rows of its window."""
+    if t == 0:
+        return 0.0
+    lo = max(0, t - w)
+    pos = np.arange(lo, t + 1)
+    seg = gen.segment_index(model, seq, t + 1)
+    m = {}
+    for l in model.band_layers:
+        rows = gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg))
+        # g[0] stands for position lo (never inside the window), g[j] for lo + j
+        g = np.array([np.nan] + [O.hidden_change(rows[i - 1], rows[i]) for i in range(1, len(pos))])
+        m[l] = O.rolling_band_mean(g, w)[-1]
+    return float(np.mean([m[l] for l in model.band_a]) - np.mean([m[l] for l in model.band_b]))
+
+
+def oracle_kv_at(model, tabs, seq, t, kind, w=64):
+    """fp64 KV-key / KV-val score of position t."""
+    pos = np.arange(max(0, t - w + 1), t + 1)
+    sp = gen.spike_flags(model, seq, t + 1)
+    X = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0 if kind == E.EPIKV_SCORE_KVKEY else 1, pos, sp))
+    return float(O.rolling_mean(np.array([O.head_variance(X[i]) for i in range(len(pos))]), w)[-1])
+
+
+def oracle_score_at(model, tabs, seq, t, kind):
+    if kind == E.EPIKV_SCORE_BANDZ:
+        return oracle_bandz_at(model, tabs, seq, t)
+    if kind == E.EPIKV_SCORE_HSVAR:
+        return oracle_hsvar_at(model, tabs, seq, t)
+    if kind in (E.EPIKV_SCORE_KVKEY, E.EPIKV_SCORE_KVVAL):
+        return oracle_kv_at(model, tabs, seq, t, kind)
+    return oracle_lag_at(model, tabs, seq, t, key_only=kind == E.EPIKV_SCORE_LAGKEY)
+
+
+def oracle_lag_at(model, tabs, seq, t, lag=16, w=64, key_only=False):
     """fp64 Lag-KV score of position t from the generator's rows it depends on."""
     t0 = max(0, t - w + 1)
     first = max(0, (t0 // lag - 1) * lag)
@@ -225,6 +272,9 @@ def oracle_lag_at(model, tabs, seq, t, lag=16, w=64):
         c = tt // lag
         if c == 0:
             u.append(0.0)
+        elif key_only:
+            lo = (c - 1) * lag - first
+            u.append(O.lag_key_token_variance(K[tt - first], K[lo:lo + lag]))
         else:
             lo = (c - 1) * lag - first
             u.append(O.lag_token_variance(K[tt - first], V[tt - first], K[lo:lo + lag], V[lo:lo + lag]))

@@ -50,7 +50,7 @@ def test_workspace_sizing_and_invalid_configs(lib):
     both = E.epikv_workspace_bytes(cfg(score_kinds=3))
     assert both > ok
     for bad in (dict(max_seqs=0), dict(head_dim=96), dict(head_dim=4), dict(hidden=4100), dict(n_band_a=0),
-                dict(z_window=0), dict(score_kinds=0), dict(score_kinds=4), dict(num_kv_heads=64),
+                dict(z_window=0), dict(score_kinds=0), dict(score_kinds=64), dict(num_kv_heads=64),
                 dict(max_new_tokens=0), dict(z_window=2000), dict(score_kinds=2, lag=0)):
         assert E.epikv_workspace_bytes(cfg(**bad)) == 0, bad
 

@@ -23,8 +23,8 @@ from paper_2606_26472_gb300.cache import KVCache
 from synth import gen, workloads as W
 from synth.device import DeviceBatchTrace, DeviceTrace, as_u16
 
-from .harness import (OracleTrace, Session, assert_scores_close, check_compaction, check_compaction_sampled,
-                      check_selection, oracle_bandz_at, oracle_lag_at)
+from .harness import (ALL_KINDS, OracleTrace, Session, assert_scores_close, check_compaction,
+                      check_compaction_sampled, check_selection, oracle_bandz_at, oracle_lag_at, oracle_score_at)
 
 pytestmark = pytest.mark.gpu
 
@@ -52,15 +52,14 @@ def _event_checks(sess, pre, kept, budgets, rng, sample_bytes, n_rows=192):
 
 def _score_samples(sess, seqs, per_seq, rng, kinds):
     for b in seqs:
-        for kind in (E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV):
+        for kind in ALL_KINDS:
             if not kinds & kind:
                 continue
             pos, sc = sess.read(b, kind)
             idx = rng.choice(len(pos), size=min(per_seq, len(pos)), replace=False)
             for i in idx:
                 t = int(pos[i])
-                ref = oracle_bandz_at(sess.m, sess.dt.tabs, b, t) if kind == E.EPIKV_SCORE_BANDZ \
-                    else oracle_lag_at(sess.m, sess.dt.tabs, b, t)
+                ref = oracle_score_at(sess.m, sess.dt.tabs, b, t, kind)
                 assert_scores_close([sc[i]], [ref], f"seq {b} kind {kind} position {t}")
 
 
@@ -122,6 +121,17 @@ def test_config2_batch8_8k_bandz(gpu_lib):
     first = wl.budgets[0] // wl.chunk            # the first step that evicts
     _run_chunked(wl, {first, 100, wl.max_len // wl.chunk - 1}, sample_bytes={0, 5}, score_seqs=range(8),
                  per_seq=6)
+
+
+def test_config2_shape_with_all_six_score_kinds(gpu_lib):
+    """The 8 x 8,192 band-z workload's shape with every score kind computed and
+    each sequence's selection driven by a different one."""
+    import dataclasses
+    wl = W.config(2)
+    pol = tuple(ALL_KINDS[b % 6] for b in range(wl.n_seq))
+    wl = dataclasses.replace(wl, kinds=63, policies=pol)
+    first = wl.budgets[0] // wl.chunk
+    _run_chunked(wl, {first, wl.max_len // wl.chunk - 1}, sample_bytes={1, 4}, score_seqs=range(6), per_seq=3)
 
 
 def test_config3_batch32_32k_lagkv_paged(gpu_lib):

@@ -9,7 +9,7 @@ from paper_2606_26472_gb300 import epikv as E
 from synth import gen, workloads as W
 from synth.device import DeviceTrace, as_u16
 
-from .harness import OracleTrace, Session, assert_scores_close, check_compaction, check_selection
+from .harness import ALL_KINDS, OracleTrace, Session, assert_scores_close, check_compaction, check_selection
 
 pytestmark = pytest.mark.gpu
 
@@ -43,7 +43,15 @@ CASES = [
     ("paged_lag", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_LAGKV, (0, 0, 20), (100, 64, 90), (16, 5, 40), 16),
     ("paged_both", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_LAGKV, (3, 0, 0), (80, 120, 50),
      (1, 9, 64), 5),
+    ("contig_all_kinds_a", E.EPIKV_LAYOUT_CONTIGUOUS, 63, (0, 2, 0), (90, 70, 110), (5, 16, 23), 16),
+    ("paged_all_kinds_b", E.EPIKV_LAYOUT_PAGED, 63, (0, 0, 9), (60, 100, 75), (32, 3, 12), 7),
 ]
+
+# the policy driving each of the three sequences' selection, per case
+POLICIES = {
+    "contig_all_kinds_a": (E.EPIKV_SCORE_HSVAR, E.EPIKV_SCORE_KVKEY, E.EPIKV_SCORE_LAGKEY),
+    "paged_all_kinds_b": (E.EPIKV_SCORE_KVVAL, E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV),
+}
 
 
 @pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks,lag", CASES, ids=[c[0] for c in CASES])
@@ -52,8 +60,9 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
     n_seq = 3
     lengths = (310, 257, 333)
     slack = 12
-    policies = [E.EPIKV_SCORE_BANDZ if (kinds & 1 and (b % 2 == 0 or kinds == 1)) else E.EPIKV_SCORE_LAGKV
-                for b in range(n_seq)]
+    policies = list(POLICIES.get(name) or
+                    [E.EPIKV_SCORE_BANDZ if (kinds & 1 and (b % 2 == 0 or kinds == 1)) else E.EPIKV_SCORE_LAGKV
+                     for b in range(n_seq)])
     max_new = max(chunks)
     T_cap = max(budgets) + slack + max_new + 1
     sess = Session(model, n_seq=n_seq, kinds=kinds, layout=layout, max_tokens=T_cap, max_new=max_new,
@@ -72,7 +81,7 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
         sess.score_update(entries)
         pre = {}
         for b, n in entries:
-            for kind in (1, 2):
+            for kind in ALL_KINDS:
                 if kinds & kind:
                     pos, sc = sess.read(b, kind)
                     new = slice(before[b], before[b] + n)
@@ -98,7 +107,7 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
 def test_chunking_invariance_and_causality(gpu_lib):
     """Scores are identical, bit for bit, however the trace is split into calls."""
     model = W.small_model(77)
-    kinds = E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_LAGKV
+    kinds = 63
     L = 200
     results = []
     for chunk in (1, 7, 64, 200):
@@ -106,11 +115,11 @@ def test_chunking_invariance_and_causality(gpu_lib):
                        max_new=chunk, prefill=(0,), policies=(1,))
         while sess.n_seen[0] < L:
             sess.score_update([(0, min(chunk, L - sess.n_seen[0]))])
-        results.append((sess.read(0, 1)[1], sess.read(0, 2)[1]))
+        results.append([sess.read(0, k)[1] for k in ALL_KINDS])
         sess.close()
     for r in results[1:]:
-        np.testing.assert_array_equal(r[0], results[0][0])
-        np.testing.assert_array_equal(r[1], results[0][1])
+        for a, b in zip(r, results[0]):
+            np.testing.assert_array_equal(a, b)
 
 
 def test_constant_signal_gives_exact_zero_and_lowest_slot_ties(gpu_lib):
