@@ -58,6 +58,9 @@ def parse():
     # the band-z kernels' workload: the 2,048-token single-sequence case, one
     # fresh sequence per step (reported for the per-kernel rooflines)
     p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k"])
+    # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
+    # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
+    p.add_argument("--kinds", type=int, default=2)
     return p.parse_args()
 
 
@@ -248,6 +251,8 @@ def run_ours(args):
     assert K % wl.block_size == 0 and C % wl.block_size == 0
     workload = WORKLOAD if (Bn, K, C) == (wl.n_seq, wl.budgets[0], wl.chunk) else \
         f"batch{Bn}_lagkv_paged16_K{K}_chunk{C}"
+    if args.kinds != E.EPIKV_SCORE_LAGKV:
+        workload += f"_kinds{args.kinds}"
     L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
     bs = wl.block_size
     T_cap = K + C
@@ -274,7 +279,8 @@ def run_ours(args):
 
     cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T_cap, max_new_tokens=C, num_layers=L, num_kv_heads=H,
                         head_dim=d, lag=wl.lag, lag_window=wl.lag_window, recency_cap=wl.recency_cap,
-                        score_kinds=E.EPIKV_SCORE_LAGKV)
+                        score_kinds=args.kinds)
+    assert args.kinds & E.EPIKV_SCORE_LAGKV and not args.kinds & (E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR)
     ws_bytes = E.epikv_workspace_bytes(cfg)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     ctx = E.epikv_init(cfg, ws, ws_bytes)
