@@ -21,8 +21,11 @@
 
 namespace epikv {
 
+#ifndef EPIKV_G_UNROLL
+#define EPIKV_G_UNROLL 2  // tokens whose rows are loaded together (measured best: 2)
+#endif
 constexpr int kGThreads = 256;
-constexpr int kGUnroll = 4;
+constexpr int kGUnroll = EPIKV_G_UNROLL;
 constexpr int kMaxTokPerCta = 16;
 
 struct BandRows {
@@ -37,7 +40,10 @@ struct BandRows {
 // of the run before it when they are consecutive, else it is loaded (from
 // the saved h_prev for a sequence's first new token).
 template <int VPT>
-__global__ void __launch_bounds__(kGThreads, (VPT >= 4 ? 2 : 4)) bandz_g_kernel(DevState st, Dims dm, BandRows rows,
+#ifndef EPIKV_G_MINB
+#define EPIKV_G_MINB 0  // 0: by register need
+#endif
+__global__ void __launch_bounds__(kGThreads, (EPIKV_G_MINB > 0 ? EPIKV_G_MINB : VPT * kGUnroll >= 16 ? 2 : 4)) bandz_g_kernel(DevState st, Dims dm, BandRows rows,
                                                             int64_t row_stride,
                                                             const int32_t* __restrict__ seq_ids,
                                                             const int32_t* __restrict__ cu_new, int n_seq,
@@ -350,7 +356,10 @@ __global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm
   }
 }
 
-constexpr int kFinTile = 32;
+#ifndef EPIKV_FIN_TILE
+#define EPIKV_FIN_TILE 16
+#endif
+constexpr int kFinTile = EPIKV_FIN_TILE;  // tokens per finalize CTA
 constexpr int kFinThreads = 256;
 constexpr int kMaxWindow = 1024;
 
