@@ -213,7 +213,8 @@ static epikv_status score_update_impl(epikv_ctx* ctx, int32_t n_seq, const int32
                                       const epikv_hidden_view* hidden, const epikv_kv_view* kv,
                                       cudaStream_t stream, int* launches) {
   if (!ctx || n_seq < 0 || n_seq > ctx->dm.S || max_new < 0 || max_new > ctx->dm.max_new) return EPIKV_EINVAL;
-  if (n_seq > 0 && (!d_seq_ids || !d_cu_new)) return EPIKV_EINVAL;
+  if (n_seq == 0) return EPIKV_OK;  // nothing to score
+  if (!d_seq_ids || !d_cu_new) return EPIKV_EINVAL;
   if (!valid_hidden(ctx, hidden)) return EPIKV_EINVAL;
   KvDev kd;
   memset(&kd, 0, sizeof(kd));
@@ -258,7 +259,8 @@ epikv_status epikv_step(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
                         const epikv_hidden_view* hidden, const epikv_kv_view* kv, int32_t* d_n_cache_out,
                         cudaStream_t stream) {
   if (!ctx || n_seq < 0 || n_seq > ctx->dm.S) return EPIKV_EINVAL;
-  if (n_seq > 0 && !d_budget) return EPIKV_EINVAL;
+  if (n_seq == 0) return EPIKV_OK;  // nothing to do
+  if (!d_budget) return EPIKV_EINVAL;
   KvDev kd;
   if (!valid_kv(ctx, kv, &kd)) return EPIKV_EINVAL;
   int launches = 0;

@@ -66,6 +66,8 @@ class DeviceTrace:
 
     def hidden(self, seq, layer, pos0, n, out, row_stride, stream=None):
         """Write rows of positions pos0..pos0+n-1 to `out` (a device pointer or tensor)."""
+        if n <= 0:
+            return
         m, tb = self.m, self.tabs
         seg = self.seg(seq, pos0 + n) if tb.seg_amp[layer] != 0 else None
         ptr = out if isinstance(out, int) else out.data_ptr()
@@ -79,6 +81,8 @@ class DeviceTrace:
     def kv(self, seq, pos0, n, slot0, k, v, *, layout, stride_layer, stride_seq=0, stride_block=0, stride_token,
            block_table=None, max_blocks=0, block_size=0, stream=None):
         """Write K and V rows of positions pos0.. to slots slot0.. of a cache view."""
+        if n <= 0:
+            return
         m = self.m
         r = load().synth_kv(m.seed & 0xFFFFFFFFFFFFFFFF, seq, pos0, n, slot0, m.num_layers, m.num_kv_heads,
                             m.head_dim, m.spike_per_10k, self.kv_scale.data_ptr(), self.kv_off.data_ptr(),
