@@ -57,7 +57,7 @@ def parse():
     p.add_argument("--chunk", type=int, default=128)
     # the band-z kernels' workload: the 2,048-token single-sequence case, one
     # fresh sequence per step (reported for the per-kernel rooflines)
-    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k"])
+    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken"])
     # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
     # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
     p.add_argument("--kinds", type=int, default=2)
@@ -552,12 +552,109 @@ def run_bandz2k(args):
     print(json.dumps(line), flush=True)
 
 
+def run_pertoken(args):
+    """The per-token regime of the 65,536-token band-z workload: 4 sequences,
+    one new token each per decode step, 15 band rows per token.  One bench
+    step = 64 decode steps, issued either call by call or as one CUDA graph
+    of 64 epikv_score_update calls (the per-step kernels are tiny, so launch
+    overhead decides the rate)."""
+    import torch
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    from synth import workloads as W
+    from synth.device import DeviceTrace
+
+    rank, local_rank, world = dist_env()
+    assert world == 1, "the per-token workload is a single-GPU measurement"
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+    wl = W.config(4)
+    m = wl.model
+    Bn, G = wl.n_seq, 64
+    n_tok = (2 * (args.warmup + args.steps) + 1) * G     # eager run, then graph run
+    nb = len(m.band_layers)
+    dt = DeviceTrace(m, dev)
+    hid = torch.empty((nb, n_tok, Bn, m.hidden), dtype=torch.bfloat16, device=dev)
+    for i, layer in enumerate(m.band_layers):
+        for b in range(Bn):
+            dt.hidden(b, layer, 0, n_tok, hid[i, :, b].data_ptr(), Bn * m.hidden)
+    cfg = E.make_config(max_seqs=Bn, max_cache_tokens=n_tok, max_new_tokens=1, n_band_a=len(m.band_a),
+                        n_band_b=len(m.band_b), score_kinds=E.EPIKV_SCORE_BANDZ)
+    ws = torch.empty(E.epikv_workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws.numel())
+    for b in range(Bn):
+        E.epikv_seq_reset(ctx, b, 0, E.EPIKV_SCORE_BANDZ)
+    seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
+    cu = torch.arange(Bn + 1, dtype=torch.int32, device=dev)
+    step_bytes = Bn * m.hidden * 2
+    bases = [hid[i].data_ptr() for i in range(nb)]
+    kv_unused = E.kv_view(hid, hid, stride_layer=0, stride_seq=0, stride_token=1024)
+
+    def view(t):
+        hv = E.epikv_hidden_view()
+        hv.row_stride = m.hidden
+        for i in range(nb):
+            hv.band_rows[i] = bases[i] + t * step_bytes
+        return hv
+
+    views = [view(t) for t in range(n_tok)]
+    stream = torch.cuda.current_stream()
+    t = 0
+    E.epikv_score_update(ctx, Bn, seq_ids, cu, 1, views[t], kv_unused)
+    t += 1
+
+    def eager_block(t0):
+        for k in range(G):
+            E.epikv_score_update(ctx, Bn, seq_ids, cu, 1, views[t0 + k], kv_unused)
+
+    def timed(run_block, t0):
+        for w in range(args.warmup):
+            run_block(t0 + w * G)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            run_block(t0 + (args.warmup + i) * G)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    ms_eager = timed(eager_block, t)
+    t += (args.warmup + args.steps) * G
+    graphs = {}
+    for blk in range(args.warmup + args.steps):     # one graph per 64-token block, captured before timing
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            eager_block(t + blk * G)
+        graphs[t + blk * G] = g
+    ms_graph = timed(lambda t0: graphs[t0].replay(), t)
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    tokens = args.steps * G * Bn
+    line = {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_graph / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "batch4_bandz_per_token_updates", "sequences": Bn, "band_layers": nb,
+                       "hidden": m.hidden, "step": "64 decode tokens per sequence",
+                       "l2": "band rows of every token resident, %.1f GiB" % (hid.numel() * 2 / 2 ** 30)},
+            "per_token_us": {"graph": 1e3 * ms_graph / (args.steps * G), "eager": 1e3 * ms_eager / (args.steps * G)},
+            "eager_value": tokens / (ms_eager / 1e3),
+            "gpu_launches": 2 * G * args.steps}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
     elif args.workload == "bandz2k":
         run_bandz2k(args)
+    elif args.workload == "pertoken":
+        run_pertoken(args)
     else:
         run_ours(args)
 
