@@ -226,8 +226,8 @@ epikv_status epikv_get_error(epikv_ctx* ctx, int32_t* code);
  * device memory -- a plugin inside an application whose memory pool owns the
  * whole GPU, an embedded caller without a device allocator, or a loop that
  * must never block on cudaMalloc -- and so cannot create the workspace that
- * epikv_init needs.  It gives the same scores epikv_score_update gives for
- * the same tokens of a fresh sequence.
+ * epikv_init needs.  Its scores agree, to fp32 rounding, with the ones
+ * epikv_score_update gives for the same tokens of a fresh sequence.
  *   kv         the caller's cache; slots 0..n-1 of `seq` hold positions 0..n-1
  *   L, H, d    layers, KV heads, head dim (d a power of two in [8, 256],
  *              H <= 32, H*d/8 <= 256)

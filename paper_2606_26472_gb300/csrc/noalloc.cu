@@ -20,9 +20,10 @@
 // (different streams, no ordering between them) race on it.
 //
 // The kernels are variants of the Lag-KV partial and finalize kernels of the
-// context path, for a sequence whose slots 0..n-1 hold positions 0..n-1; they
-// use the same arithmetic in the same order, so the scores equal the ones
-// epikv_score_update produces for the same tokens.
+// context path, for a sequence whose slots 0..n-1 hold positions 0..n-1.  They
+// take each head's variance in two passes (mean, then squared deviations),
+// where the context path uses shifted moments in one pass, so the scores agree
+// with epikv_score_update's to fp32 rounding, not bit for bit.
 #include <mutex>
 
 #include "common.cuh"
