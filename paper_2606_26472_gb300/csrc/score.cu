@@ -169,7 +169,13 @@ __global__ void __launch_bounds__(kGThreads, (EPIKV_G_MINB > 0 ? EPIKV_G_MINB : 
   }
 }
 
-constexpr int kLagSeg = 16;     // tokens per segment (never crosses a chunk boundary)
+#ifndef EPIKV_LAG_SEG
+#define EPIKV_LAG_SEG 8
+#endif
+#ifndef EPIKV_LAG_MINB
+#define EPIKV_LAG_MINB 3  // caps registers at 80 (measured best with 8-token segments)
+#endif
+constexpr int kLagSeg = EPIKV_LAG_SEG;  // tokens per segment (never crosses a chunk boundary)
 constexpr int kLagOffs = 256;   // slot offsets looked up per group of tokens
 
 __device__ __forceinline__ uint32_t bf16x2_min(uint32_t a, uint32_t b) {
@@ -207,7 +213,7 @@ __device__ __forceinline__ void prev_range(const uint4& pmn, const uint4& pmx, f
 // is taken from the moments of y = x~ - 1/2 (x~ in [0, 1] inside the range),
 // one two-value group reduction per token.
 template <int LH>
-__global__ void __launch_bounds__(256) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
+__global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
                                                              const int32_t* __restrict__ seq_ids,
                                                              const int32_t* __restrict__ cu_new,
                                                              int max_new) {
