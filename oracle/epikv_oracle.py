@@ -37,6 +37,15 @@ R12 KV-key / KV-val variance: the population variance over the head
     over (layer, head), then the rolling mean of R10; every position has a
     value (no chunk 0 exception).
 R13 lag-kv-key: Lag-KV (R10) with the key term only.
+R18 chunk-level selection (named as future work in Sec. 5, after ChunkKV's
+    contiguous chunks of Sec. 2): positions fall into fixed chunks
+    floor(pos / C); a chunk's score is the mean of the frozen scores of its
+    members that are candidates (prefill and recency slots are not members),
+    summed left to right in float32 and divided by the member count in
+    float32, the precision the ranking is decided in on both sides; chunks
+    rank by that score (R8's order: NaN lowest, -0 == +0, ties to the
+    earlier chunk) and fill the M candidate places whole, in rank order; the
+    first chunk that does not fit gives its lowest slots.  C = 1 is R7/R8.
 """
 from __future__ import annotations
 
@@ -231,6 +240,56 @@ def select_kept(scores, K, prefill=0, recency_cap=128):
     return sorted(kept)
 
 
+def chunk_scores(scores, positions, candidates, chunk):
+    """Float32 mean score of every chunk of candidate slots (R18).
+
+    Returns {chunk id: (mean, [member slots in slot order])}; chunk id =
+    floor(position / chunk).
+    """
+    members = {}
+    for i in candidates:
+        members.setdefault(int(positions[i]) // chunk, []).append(i)
+    out = {}
+    for c, slots in members.items():
+        s = np.float32(0.0)
+        for i in slots:                                   # left to right
+            s = np.float32(s + np.float32(scores[i]))
+        out[c] = (np.float32(s / np.float32(len(slots))), slots)
+    return out
+
+
+def select_kept_chunked(scores, positions, K, prefill=0, recency_cap=128, chunk=1):
+    """Ascending kept slot list under chunk-level selection (R18).
+
+    Same protected set and budget split as ``select_kept``; the M candidate
+    places go to whole position chunks in the order of their mean score,
+    the first chunk that does not fit contributing its lowest slots.
+    """
+    scores = np.asarray(scores, dtype=np.float64)
+    n = scores.shape[0]
+    if n <= K:
+        return list(range(n))
+    P = min(prefill, n)
+    R = min(recency_window(K, recency_cap), max(0, K - P))
+    M = max(0, K - P - R)
+    candidates = list(range(P, n - R))
+    chunks = chunk_scores(scores, positions, candidates, chunk)
+
+    def rank(c):  # NaN last, higher mean first, earlier chunk first
+        s = float(chunks[c][0])
+        return (1, 0.0, c) if np.isnan(s) else (0, -s, c)
+
+    best = []
+    for c in sorted(chunks, key=rank):
+        slots = chunks[c][1]
+        take = min(len(slots), M - len(best))
+        best.extend(slots[:take])
+        if len(best) == M:
+            break
+    kept = set(range(P)) | set(range(n - R, n)) | set(best)
+    return sorted(kept)
+
+
 # --------------------------------------------------------------------------
 # App. H -- rebuild the cache from the kept entries, in order
 # --------------------------------------------------------------------------
@@ -239,19 +298,24 @@ def compact(rows, kept):
     return np.asarray(rows)[np.asarray(kept, dtype=np.int64)]
 
 
-def simulate_decode(scores, length, chunk, K, trigger, prefill=0, recency_cap=128):
+def simulate_decode(scores, length, chunk, K, trigger, prefill=0, recency_cap=128, select_chunk=1):
     """Replay one sequence's decode: append ``chunk`` tokens at a time and
     evict whenever the cache holds more than ``trigger`` tokens.
 
-    scores: frozen score of every position (R6).  Returns the list of events
-    as (positions before, positions after) and the final position list.
+    scores: frozen score of every position (R6).  ``select_chunk`` > 1 uses
+    chunk-level selection (R18).  Returns the list of events as (positions
+    before, positions after) and the final position list.
     """
     cache = []
     events = []
     for start in range(0, length, chunk):
         cache.extend(range(start, min(length, start + chunk)))
         if len(cache) > trigger:
-            kept = select_kept([scores[p] for p in cache], K, prefill, recency_cap)
+            if select_chunk > 1:
+                kept = select_kept_chunked([scores[p] for p in cache], cache, K, prefill, recency_cap,
+                                           select_chunk)
+            else:
+                kept = select_kept([scores[p] for p in cache], K, prefill, recency_cap)
             after = [cache[i] for i in kept]
             events.append((list(cache), after))
             cache = list(after)

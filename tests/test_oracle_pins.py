@@ -333,6 +333,131 @@ def test_simulate_decode_keeps_structure():
     assert len(final) <= 256 + 15
 
 
+
+# ------------------------------------- chunk-level selection (Sec. 5 future work)
+def _golden_chunk_cases():
+    pos = score = None
+    cases = []
+    with open(os.path.join(GOLDEN, "chunk_select_hand_example.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            head, *rest = line.split()
+            if head == "pos":
+                pos = [int(x) for x in rest]
+            elif head == "score":
+                score = [float(x) for x in rest]
+            elif head == "case":
+                K, P, cap, C = (int(x) for x in rest[:4])
+                cases.append((K, P, cap, C, [int(x) for x in rest[5:]]))
+    return pos, score, cases
+
+
+def test_chunked_select_hand_example():
+    pos, score, cases = _golden_chunk_cases()
+    assert len(cases) == 3
+    for K, P, cap, C, kept in cases:
+        assert O.select_kept_chunked(score, pos, K, P, cap, C) == kept
+
+
+def test_chunked_select_with_unit_chunks_is_the_token_rule():
+    rng = np.random.default_rng(21)
+    for trial in range(200):
+        n = int(rng.integers(1, 60))
+        s = rng.integers(-3, 4, size=n).astype(np.float64)
+        if trial % 3 == 0:
+            s[rng.integers(0, n, size=3)] = np.nan
+        if trial % 4 == 0:
+            s[s == 0] = -0.0
+        pos = np.cumsum(rng.integers(1, 4, size=n)) - 1
+        K, P, cap = int(rng.integers(1, 40)), int(rng.integers(0, 6)), int(rng.integers(0, 10))
+        assert O.select_kept_chunked(s, pos, K, P, cap, 1) == O.select_kept(s, K, P, cap)
+
+
+def _brute_chunked(s, pos, K, P, cap, C):
+    """Every M-subset of the candidates is tried; the kept one is the unique
+    subset whose every member outranks every other candidate when a slot is
+    valued by its chunk's exact (rational) mean, NaN lowest, lower slot on
+    ties -- whole chunks in rank order, the boundary chunk's lowest slots."""
+    from fractions import Fraction
+    n = len(s)
+    if n <= K:
+        return list(range(n))
+    P = min(P, n)
+    R = min(min(cap, K // 4), max(0, K - P))
+    M = max(0, K - P - R)
+    cand = list(range(P, n - R))
+    val = {}
+    for i in cand:
+        mates = [j for j in cand if pos[j] // C == pos[i] // C]
+        if any(math.isnan(s[j]) for j in mates):
+            val[i] = None
+        else:
+            val[i] = sum(Fraction(s[j]) for j in mates) / len(mates)
+
+    def better(i, j):
+        a, b = val[i], val[j]
+        if a is None or b is None:
+            return (a is not None) or (b is None and i < j)
+        return a > b or (a == b and i < j)
+
+    valid = [S for S in itertools.combinations(cand, M)
+             if all(better(i, j) for i in S for j in cand if j not in S)]
+    assert len(valid) == 1
+    return sorted(set(range(P)) | set(range(n - R, n)) | set(valid[0]))
+
+
+def test_chunked_select_equals_brute_force_on_tiny_inputs():
+    rng = np.random.default_rng(22)
+    for trial in range(300):
+        n = int(rng.integers(1, 12))
+        K = int(rng.integers(1, 10))
+        P = int(rng.integers(0, 3))
+        cap = int(rng.integers(0, 4))
+        C = int(rng.integers(2, 5))
+        pos = list(np.cumsum(rng.integers(1, 4, size=n)) - 1)
+        s = (rng.integers(-4, 5, size=n) / 2.0).astype(np.float64)   # exact halves, many ties
+        if trial % 6 == 0:
+            s[rng.integers(0, n)] = np.nan
+        assert O.select_kept_chunked(s, pos, K, P, cap, C) == _brute_chunked(list(s), pos, K, P, cap, C)
+
+
+def test_chunked_select_structure_on_decode_histories():
+    """Along a decode with evictions every 16 tokens: K kept, prefill and the
+    recency window kept, every candidate chunk kept whole or dropped whole
+    except one, whose kept members are its lowest slots, and no dropped chunk
+    outranks a kept one."""
+    rng = np.random.default_rng(23)
+    for C in (2, 5, 16):
+        L, K, P = 900, 160, 6
+        s = rng.normal(size=L)
+        events, final = O.simulate_decode(s, L, 16, K, K + 15, prefill=P, select_chunk=C)
+        assert len(events) > 10
+        for before, after in events:
+            n = len(before)
+            R = min(128, K // 4)
+            assert len(after) == K and after == sorted(after)
+            assert after[:P] == list(range(P)) and after[-R:] == before[-R:]
+            kept = set(after)
+            chunks = {}
+            for p in before[P:n - R]:
+                chunks.setdefault(p // C, []).append(p)
+            partial = 0
+            kept_means, dropped_means = [], []
+            for c, members in chunks.items():
+                k = [p for p in members if p in kept]
+                m = math.fsum(s[p] for p in members) / len(members)
+                if k and len(k) < len(members):
+                    partial += 1
+                    assert k == members[:len(k)]
+                if k:
+                    kept_means.append(m)
+                else:
+                    dropped_means.append(m)
+            assert partial <= 1
+            if kept_means and dropped_means:
+                assert min(kept_means) >= max(dropped_means) - 1e-6
+
 # ------------------------------------------- the other attention-free variants
 def test_hsvar_closed_forms():
     # a walk with constant step a in Band A and b in Band B: g-bar = a, b
