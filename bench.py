@@ -61,6 +61,9 @@ def parse():
     # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
     # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
     p.add_argument("--kinds", type=int, default=2)
+    # chunk-level selection at the 32k workload: position chunks of this many
+    # tokens (1 = the paper's token-level selection)
+    p.add_argument("--select-chunk", type=int, default=1)
     return p.parse_args()
 
 
@@ -253,6 +256,8 @@ def run_ours(args):
         f"batch{Bn}_lagkv_paged16_K{K}_chunk{C}"
     if args.kinds != E.EPIKV_SCORE_LAGKV:
         workload += f"_kinds{args.kinds}"
+    if args.select_chunk > 1:
+        workload += f"_selectchunk{args.select_chunk}"
     L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
     bs = wl.block_size
     T_cap = K + C
@@ -279,7 +284,7 @@ def run_ours(args):
 
     cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T_cap, max_new_tokens=C, num_layers=L, num_kv_heads=H,
                         head_dim=d, lag=wl.lag, lag_window=wl.lag_window, recency_cap=wl.recency_cap,
-                        score_kinds=args.kinds)
+                        score_kinds=args.kinds, select_chunk=args.select_chunk)
     assert args.kinds & E.EPIKV_SCORE_LAGKV and not args.kinds & (E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR)
     ws_bytes = E.epikv_workspace_bytes(cfg)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
@@ -432,7 +437,8 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": workload, "sequences": Bn, "context": 32768, "budget_K": K, "chunk": C,
                    "layers": L, "kv_heads": H, "head_dim": d, "kv_dtype": "bf16", "layout": "paged16_shuffled",
-                   "score": "lagkv_lag16_w64", "parallelism": f"replicas{world}",
+                   "score": "lagkv_lag16_w64", "select_chunk": args.select_chunk,
+                   "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
         "compaction_gbs": ach,
         "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,

@@ -99,6 +99,14 @@ typedef struct {
   int32_t lag_window;       /* rolling-mean window of the K/V scores (64), 1..1024 */
   int32_t recency_cap;      /* recency window R = min(recency_cap, K/4) (App. D: 128) */
   int32_t score_kinds;      /* EPIKV_SCORE_* mask (1..63) computed by every update */
+  int32_t select_chunk;     /* C, 0..65536 (0 reads as 1).  1: the paper's token-level top-K.
+                             * C > 1: chunk-level selection, which the paper names as future
+                             * work (Sec. 5, after ChunkKV's contiguous chunks, Sec. 2): the
+                             * candidates fall into fixed position chunks floor(pos / C), a
+                             * chunk scores the fp32 mean of its candidate members' scores
+                             * (summed in slot order), and whole chunks fill the candidate
+                             * budget in rank order (NaN lowest, ties to the earlier chunk);
+                             * the first chunk that does not fit keeps its lowest slots. */
 } epikv_config;
 
 /* New hidden-state rows of one update call (Sec. 3.1: the per-layer hidden

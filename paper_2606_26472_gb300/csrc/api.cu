@@ -42,6 +42,7 @@ bool valid_config(const epikv_config* c) {
   if (c->max_new_tokens < 1 || c->max_new_tokens > (1 << 20)) return false;
   if (c->score_kinds < 1 || c->score_kinds > 63) return false;
   if (c->recency_cap < 0) return false;
+  if (c->select_chunk < 0 || c->select_chunk > 65536) return false;
   if (c->num_layers < 1 || c->num_kv_heads < 1 || c->num_kv_heads > 32) return false;
   if (!is_pow2(c->head_dim) || c->head_dim < 8 || c->head_dim > 256) return false;
   if (c->num_kv_heads * c->head_dim / 8 > 256) return false;
@@ -68,6 +69,7 @@ Dims make_dims(const epikv_config* c) {
   d.d = c->head_dim;
   d.kinds = c->score_kinds;
   d.recency_cap = c->recency_cap;
+  d.select_chunk = c->select_chunk > 1 ? c->select_chunk : 1;
   const bool bz = c->score_kinds & kBandKinds, lg = c->score_kinds & kKvKinds;
   d.D = bz ? c->hidden : 0;
   d.nA = bz ? c->n_band_a : 0;
@@ -119,6 +121,7 @@ size_t carve(const Dims& d, DevState* st, char* base) {
   if (d.kinds & kRawKinds) st->raw_part = (float*)take(S * (size_t)d.max_new * 2 * d.L * 4);
   for (int q = 0; q < 4; ++q)
     if (d.kinds & kv_kind(q)) st->u_ring[q] = (float*)take(S * (size_t)d.G * 4);
+  if (d.select_chunk > 1) st->ckey = (uint32_t*)take(S * T * 4);
   return align_up(off, 256);
 }
 

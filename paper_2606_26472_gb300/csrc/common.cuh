@@ -53,11 +53,12 @@ struct DevState {
   float* u_ring[4];        // [S][G] per K/V kind (kv_kind order): u by position (mod G)
   int32_t* kept;           // [S][T] kept lists of epikv_step
   int32_t* n_kept;         // [S]
+  uint32_t* ckey;          // [S][T] chunk-level selection: each candidate slot's chunk key (C > 1 only)
 };
 
 struct Dims {
   int S, T, max_new, L, H, d, D, nA, nB, G;
-  int z_window, lag, lag_window, recency_cap, kinds;
+  int z_window, lag, lag_window, recency_cap, kinds, select_chunk;
   float z_eps, lag_eps;
 };
 

@@ -9,6 +9,16 @@
 // scans emit the kept list in ascending slot order.  The slot metadata
 // (scores of every kind and positions) is then compacted in place, which is
 // safe in increasing order because kept[i] >= i.
+//
+// Chunk-level selection (select_chunk = C > 1; the paper names chunk-level
+// scoring as future work, Sec. 5): a first pass gives every candidate slot the
+// key of its position chunk floor(pos / C), the fp32 mean of the chunk's
+// candidate scores summed in slot order by the thread that owns the chunk's
+// first slot.  Chunks are runs of consecutive slots (positions increase with
+// the slot), so the unchanged selection on those keys -- larger keys first,
+// equal keys lowest slot first -- keeps whole chunks in rank order, ties to
+// the earlier chunk, and the lowest slots of the first chunk that does not
+// fit.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -68,6 +78,7 @@ __device__ __forceinline__ int block_min(int v, int* sh) {
   return r;
 }
 
+template <bool kChunked>
 __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims dm,
                                                              const int32_t* __restrict__ seq_ids,
                                                              const int32_t* __restrict__ budget,
@@ -113,6 +124,24 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   const float* __restrict__ sc = st.score[kind_index(st.policy[seq])] + (size_t)seq * dm.T;
   int32_t* out = kept_out + (size_t)b * kept_stride;
 
+  // ---- chunk keys (chunk-level selection only)
+  uint32_t* __restrict__ ck = kChunked ? st.ckey + (size_t)seq * dm.T : nullptr;
+  if (kChunked) {
+    const int C = dm.select_chunk;
+    const int32_t* __restrict__ pz = st.pos + (size_t)seq * dm.T;
+    for (int i = c0 + tid; i < c1; i += kSelThreads) {
+      const int c = pz[i] / C;
+      if (i > c0 && pz[i - 1] / C == c) continue;  // not the chunk's first candidate
+      float s = 0.f;
+      int j = i;
+      for (; j < c1 && pz[j] / C == c; ++j) s = __fadd_rn(s, sc[j]);  // at most C members
+      const uint32_t k = order_key(__fdiv_rn(s, (float)(j - i)));
+      for (int q = i; q < j; ++q) ck[q] = k;
+    }
+    __syncthreads();
+  }
+  auto key_at = [&](int i) -> uint32_t { return kChunked ? ck[i] : order_key(sc[i]); };
+
   __shared__ uint32_t hist[256];
   __shared__ uint32_t sh_prefix, sh_mask, sh_remaining;
   __shared__ int sh_scan[32];
@@ -127,7 +156,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
       __syncthreads();
       const uint32_t prefix = sh_prefix, mask = sh_mask;
       for (int i = c0 + tid; i < c1; i += kSelThreads) {
-        const uint32_t k = order_key(sc[i]);
+        const uint32_t k = key_at(i);
         if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
       }
       __syncthreads();
@@ -170,7 +199,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   const int per = (n + kSelThreads - 1) / kSelThreads;
   const int a = min(n, tid * per), e = min(n, a + per);
   int eq_local = 0;
-  for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (order_key(sc[i]) == theta);
+  for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (key_at(i) == theta);
   int tot;
   const int eq_base = block_exclusive_scan(eq_local, &tot, sh_scan);
 
@@ -180,7 +209,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
     for (int i = a; i < e; ++i) {
       bool keep = (i < c0) || (i >= c1);
       if (!keep) {
-        const uint32_t k = order_key(sc[i]);
+        const uint32_t k = key_at(i);
         keep = k > theta || (k == theta && eqs++ < need_eq);
       }
       if (keep) ++keep_local; else first_ev = min(first_ev, i);
@@ -193,7 +222,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
     for (int i = a; i < e; ++i) {
       bool keep = (i < c0) || (i >= c1);
       if (!keep) {
-        const uint32_t k = order_key(sc[i]);
+        const uint32_t k = key_at(i);
         keep = k > theta || (k == theta && eqs++ < need_eq);
       }
       if (keep) out[o++] = i;
@@ -236,7 +265,12 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
                           const int32_t* budget, const int32_t* trigger, int32_t* kept, int kept_stride,
                           int32_t* n_kept, cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
-  select_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride, n_kept);
+  if (dm.select_chunk > 1)
+    select_kernel<true><<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
+                                                           n_kept);
+  else
+    select_kernel<false><<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
+                                                            n_kept);
   ++*launches;
   return cudaGetLastError();
 }

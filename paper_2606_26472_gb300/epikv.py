@@ -23,7 +23,8 @@ class epikv_config(C.Structure):
                 ("num_layers", C.c_int32), ("num_kv_heads", C.c_int32), ("head_dim", C.c_int32),
                 ("hidden", C.c_int32), ("n_band_a", C.c_int32), ("n_band_b", C.c_int32),
                 ("z_window", C.c_int32), ("z_eps", C.c_float), ("lag", C.c_int32), ("lag_eps", C.c_float),
-                ("lag_window", C.c_int32), ("recency_cap", C.c_int32), ("score_kinds", C.c_int32)]
+                ("lag_window", C.c_int32), ("recency_cap", C.c_int32), ("score_kinds", C.c_int32),
+                ("select_chunk", C.c_int32)]
 
 
 class epikv_hidden_view(C.Structure):
@@ -114,9 +115,10 @@ def _stream(s):
 
 def make_config(*, max_seqs, max_cache_tokens, max_new_tokens, num_layers=32, num_kv_heads=8, head_dim=128,
                 hidden=4096, n_band_a=7, n_band_b=8, z_window=64, z_eps=1e-6, lag=16, lag_eps=1e-6,
-                lag_window=64, recency_cap=128, score_kinds=EPIKV_SCORE_BANDZ):
+                lag_window=64, recency_cap=128, score_kinds=EPIKV_SCORE_BANDZ, select_chunk=1):
     return epikv_config(max_seqs, max_cache_tokens, max_new_tokens, num_layers, num_kv_heads, head_dim, hidden,
-                        n_band_a, n_band_b, z_window, z_eps, lag, lag_eps, lag_window, recency_cap, score_kinds)
+                        n_band_a, n_band_b, z_window, z_eps, lag, lag_eps, lag_window, recency_cap, score_kinds,
+                        select_chunk)
 
 
 def hidden_view(band_rows, row_stride):

@@ -6,7 +6,8 @@ Acceptance rules:
 * kept sets: the oracle's selection run on the GPU's own fp32 scores must
   equal the GPU's kept list exactly; against the oracle's fp64 scores, a slot
   may differ only if its reference score is within the score tolerance of the
-  M-th candidate's score (a threshold tie);
+  M-th candidate's score (a threshold tie); under chunk-level selection the
+  same holds for the slot's chunk mean and the boundary chunk's mean;
 * compacted K/V: byte-identical to the generator's rows of the kept positions.
 """
 from __future__ import annotations
@@ -71,20 +72,21 @@ class Session:
 
     def __init__(self, model, *, n_seq, kinds, layout, max_tokens, max_new, prefill, policies,
                  z_window=64, lag=16, lag_window=64, recency_cap=128, block_size=16, shuffle_blocks=True,
-                 device="cuda"):
+                 select_chunk=1, device="cuda"):
         self.m = model
         self.n_seq = n_seq
         self.kinds = kinds
         self.prefill = list(prefill)
         self.policies = list(policies)
         self.recency_cap = recency_cap
+        self.select_chunk = select_chunk
         self.max_new = max_new
         self.dt = DeviceTrace(model, device)
         self.cfg = E.make_config(max_seqs=n_seq, max_cache_tokens=max_tokens, max_new_tokens=max_new,
                                  num_layers=model.num_layers, num_kv_heads=model.num_kv_heads,
                                  head_dim=model.head_dim, hidden=model.hidden, n_band_a=len(model.band_a),
                                  n_band_b=len(model.band_b), z_window=z_window, lag=lag, lag_window=lag_window,
-                                 recency_cap=recency_cap, score_kinds=kinds)
+                                 recency_cap=recency_cap, score_kinds=kinds, select_chunk=select_chunk)
         nbytes = E.epikv_workspace_bytes(self.cfg)
         assert nbytes > 0
         self.ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
@@ -191,10 +193,20 @@ class Session:
         E.epikv_destroy(self.ctx)
 
 
-def check_selection(kept_gpu, pos_pre, sc_gpu_pre, sc_ref_pre, K, P, cap):
+def oracle_kept(sc, pos, K, P, cap, chunk=1):
+    """The oracle's kept slots: token-level, or chunk-level for chunk > 1."""
+    if chunk > 1:
+        return O.select_kept_chunked(np.asarray(sc, np.float64), pos, K, P, cap, chunk)
+    return O.select_kept(np.asarray(sc, np.float64), K, P, cap)
+
+
+def check_selection(kept_gpu, pos_pre, sc_gpu_pre, sc_ref_pre, K, P, cap, chunk=1):
     """Exact check on the GPU's own scores + threshold-tie check on fp64."""
-    exp = O.select_kept(sc_gpu_pre.astype(np.float64), K, P, cap)
+    exp = oracle_kept(sc_gpu_pre, pos_pre, K, P, cap, chunk)
     assert list(kept_gpu) == exp, "selection differs from the oracle run on the GPU's scores"
+    if chunk > 1:
+        _check_chunk_ties(kept_gpu, pos_pre, sc_ref_pre, K, P, cap, chunk)
+        return
     ref = O.select_kept(sc_ref_pre, K, P, cap)
     if list(kept_gpu) != ref:
         n = len(sc_ref_pre)
@@ -207,6 +219,31 @@ def check_selection(kept_gpu, pos_pre, sc_gpu_pre, sc_ref_pre, K, P, cap):
         for i in diff:
             assert abs(sc_ref_pre[i] - theta) <= TOL * max(1.0, abs(theta)), \
                 f"slot {i} differs from the fp64 selection away from the threshold"
+
+
+def _check_chunk_ties(kept_gpu, pos_pre, sc_ref_pre, K, P, cap, chunk):
+    """Against fp64 scores, chunk-level: a slot may differ only if its chunk's
+    mean is within the tolerance of the boundary chunk's mean."""
+    ref = O.select_kept_chunked(sc_ref_pre, pos_pre, K, P, cap, chunk)
+    diff = set(kept_gpu) ^ set(ref)
+    if not diff:
+        return
+    n = len(sc_ref_pre)
+    Pp = min(P, n)
+    R = min(min(cap, K // 4), max(0, K - Pp))
+    M = max(0, K - Pp - R)
+    chunks = O.chunk_scores(sc_ref_pre, pos_pre, range(Pp, n - R), chunk)
+    mean_of = {i: float(m) for m, slots in chunks.values() for i in slots}
+    order = sorted(chunks, key=lambda c: (np.isnan(chunks[c][0]), -chunks[c][0], c))
+    filled, theta = 0, np.inf
+    for c in order:
+        filled += len(chunks[c][1])
+        if filled >= M:
+            theta = float(chunks[c][0])
+            break
+    for i in diff:
+        assert abs(mean_of[i] - theta) <= TOL * max(1.0, abs(theta)), \
+            f"slot {i} differs from the fp64 chunk selection away from the threshold"
 
 
 def oracle_bandz_at(model, tabs, seq, t, w=64):

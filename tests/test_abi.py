@@ -49,9 +49,13 @@ def test_workspace_sizing_and_invalid_configs(lib):
     assert ok > 0 and ok % 256 == 0
     both = E.epikv_workspace_bytes(cfg(score_kinds=3))
     assert both > ok
+    # chunk-level selection adds one key per slot; 0 and 1 are the token rule
+    assert E.epikv_workspace_bytes(cfg(select_chunk=0)) == E.epikv_workspace_bytes(cfg(select_chunk=1)) == ok
+    assert E.epikv_workspace_bytes(cfg(select_chunk=16)) >= ok + 4 * 4 * 1024
     for bad in (dict(max_seqs=0), dict(head_dim=96), dict(head_dim=4), dict(hidden=4100), dict(n_band_a=0),
                 dict(z_window=0), dict(score_kinds=0), dict(score_kinds=64), dict(num_kv_heads=64),
-                dict(max_new_tokens=0), dict(z_window=2000), dict(score_kinds=2, lag=0)):
+                dict(max_new_tokens=0), dict(z_window=2000), dict(score_kinds=2, lag=0),
+                dict(select_chunk=-1), dict(select_chunk=65537)):
         assert E.epikv_workspace_bytes(cfg(**bad)) == 0, bad
 
 

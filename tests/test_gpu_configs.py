@@ -24,7 +24,8 @@ from synth import gen, workloads as W
 from synth.device import DeviceBatchTrace, DeviceTrace, as_u16
 
 from .harness import (ALL_KINDS, OracleTrace, Session, assert_scores_close, check_compaction,
-                      check_compaction_sampled, check_selection, oracle_bandz_at, oracle_lag_at, oracle_score_at)
+                      check_compaction_sampled, check_selection, oracle_bandz_at, oracle_kept, oracle_lag_at,
+                      oracle_score_at)
 
 pytestmark = pytest.mark.gpu
 
@@ -42,7 +43,7 @@ class _CacheProbe:
 def _event_checks(sess, pre, kept, budgets, rng, sample_bytes, n_rows=192):
     for b, kl in kept.items():
         pos, sc = pre[b]
-        exp = O.select_kept(sc.astype(np.float64), budgets[b], sess.prefill[b], sess.recency_cap)
+        exp = oracle_kept(sc, pos, budgets[b], sess.prefill[b], sess.recency_cap, sess.select_chunk)
         assert list(kl) == exp, f"seq {b}: selection differs from the oracle on the GPU's scores"
         pos_after, _ = sess.read(b, sess.policies[b])
         np.testing.assert_array_equal(pos_after, pos[kl])
@@ -63,12 +64,12 @@ def _score_samples(sess, seqs, per_seq, rng, kinds):
                 assert_scores_close([sc[i]], [ref], f"seq {b} kind {kind} position {t}")
 
 
-def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq):
+def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq, select_chunk=1):
     m = wl.model
     rng = np.random.default_rng(wl.model.seed)
     K = wl.budgets[0]
     sess = Session(m, n_seq=wl.n_seq, kinds=wl.kinds, layout=wl.layout, max_tokens=K + wl.chunk,
-                   max_new=wl.chunk, prefill=[0] * wl.n_seq, policies=wl.policies)
+                   max_new=wl.chunk, prefill=[0] * wl.n_seq, policies=wl.policies, select_chunk=select_chunk)
     budgets = list(wl.budgets)
     triggers = [budgets[b] + wl.trigger_slack[b] for b in range(wl.n_seq)]
     n_steps = wl.max_len // wl.chunk
@@ -121,6 +122,15 @@ def test_config2_batch8_8k_bandz(gpu_lib):
     first = wl.budgets[0] // wl.chunk            # the first step that evicts
     _run_chunked(wl, {first, 100, wl.max_len // wl.chunk - 1}, sample_bytes={0, 5}, score_seqs=range(8),
                  per_seq=6)
+
+
+def test_config2_shape_with_chunk_level_selection(gpu_lib):
+    """The 8 x 8,192 band-z workload with chunk-level selection (16-position
+    chunks), every step through epikv_step except the sampled events."""
+    wl = W.config(2)
+    first = wl.budgets[0] // wl.chunk
+    _run_chunked(wl, {first, 77, wl.max_len // wl.chunk - 1}, sample_bytes={3}, score_seqs=(2,), per_seq=3,
+                 select_chunk=16)
 
 
 def test_config2_shape_with_all_six_score_kinds(gpu_lib):

@@ -38,13 +38,20 @@ def test_generator_device_twin_is_bit_identical(gpu_lib):
 
 
 CASES = [
-    # layout, kinds, prefill, budgets, chunk pattern, lag
-    ("contig_bandz", E.EPIKV_LAYOUT_CONTIGUOUS, E.EPIKV_SCORE_BANDZ, (0, 5, 0), (100, 60, 130), (7, 1, 33), 16),
-    ("paged_lag", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_LAGKV, (0, 0, 20), (100, 64, 90), (16, 5, 40), 16),
+    # layout, kinds, prefill, budgets, new-token pattern, lag, selection chunk C
+    ("contig_bandz", E.EPIKV_LAYOUT_CONTIGUOUS, E.EPIKV_SCORE_BANDZ, (0, 5, 0), (100, 60, 130), (7, 1, 33), 16, 1),
+    ("paged_lag", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_LAGKV, (0, 0, 20), (100, 64, 90), (16, 5, 40), 16, 1),
     ("paged_both", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_LAGKV, (3, 0, 0), (80, 120, 50),
-     (1, 9, 64), 5),
-    ("contig_all_kinds_a", E.EPIKV_LAYOUT_CONTIGUOUS, 63, (0, 2, 0), (90, 70, 110), (5, 16, 23), 16),
-    ("paged_all_kinds_b", E.EPIKV_LAYOUT_PAGED, 63, (0, 0, 9), (60, 100, 75), (32, 3, 12), 7),
+     (1, 9, 64), 5, 1),
+    ("contig_all_kinds_a", E.EPIKV_LAYOUT_CONTIGUOUS, 63, (0, 2, 0), (90, 70, 110), (5, 16, 23), 16, 1),
+    ("paged_all_kinds_b", E.EPIKV_LAYOUT_PAGED, 63, (0, 0, 9), (60, 100, 75), (32, 3, 12), 7, 1),
+    # chunk-level selection
+    ("contig_bandz_chunk4", E.EPIKV_LAYOUT_CONTIGUOUS, E.EPIKV_SCORE_BANDZ, (0, 5, 0), (100, 60, 130), (7, 1, 33),
+     16, 4),
+    ("paged_lag_chunk16", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_LAGKV, (0, 0, 20), (100, 64, 90), (16, 5, 40), 16,
+     16),
+    ("paged_both_chunk3", E.EPIKV_LAYOUT_PAGED, E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_LAGKV, (3, 0, 0),
+     (80, 120, 50), (1, 9, 64), 5, 3),
 ]
 
 # the policy driving each of the three sequences' selection, per case
@@ -54,8 +61,9 @@ POLICIES = {
 }
 
 
-@pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks,lag", CASES, ids=[c[0] for c in CASES])
-def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chunks, lag):
+@pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks,lag,select_chunk", CASES,
+                         ids=[c[0] for c in CASES])
+def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chunks, lag, select_chunk):
     model = W.small_model(1000 + len(name))
     n_seq = 3
     lengths = (310, 257, 333)
@@ -66,7 +74,7 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
     max_new = max(chunks)
     T_cap = max(budgets) + slack + max_new + 1
     sess = Session(model, n_seq=n_seq, kinds=kinds, layout=layout, max_tokens=T_cap, max_new=max_new,
-                   prefill=prefill, policies=policies, lag=lag)
+                   prefill=prefill, policies=policies, lag=lag, select_chunk=select_chunk)
     refs = [OracleTrace(model, sess.dt.tabs, b, lengths[b], kinds, lag=lag) for b in range(n_seq)]
     events = 0
     step = 0
@@ -95,7 +103,8 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
         for b, kl in kept.items():
             events += 1
             pos, sc = pre[b]
-            check_selection(kl, pos, sc, refs[b].scores[policies[b]][pos], budgets[b], prefill[b], 128)
+            check_selection(kl, pos, sc, refs[b].scores[policies[b]][pos], budgets[b], prefill[b], 128,
+                            select_chunk)
             pos_after, _ = sess.read(b, policies[b])
             np.testing.assert_array_equal(pos_after, pos[kl])
             check_compaction(sess, b, pos_after)
