@@ -46,6 +46,13 @@ R18 chunk-level selection (named as future work in Sec. 5, after ChunkKV's
     rank by that score (R8's order: NaN lowest, -0 == +0, ties to the
     earlier chunk) and fill the M candidate places whole, in rank order; the
     first chunk that does not fit gives its lowest slots.  C = 1 is R7/R8.
+R19 per-layer budgets (named as future work in Sec. 5, after PyramidKV's
+    per-layer allocation of Sec. 2): layer l has its own budget K_l and its
+    own cache, and evicts it by R7/R8 on its own, except that every layer
+    uses the same recency window R = min(cap, floor(K_min / 4)), shrunk to
+    max(0, K_min - P), K_min the smallest budget, and M_l = max(0, K_l - P -
+    R); all layers evict at the same events, when the largest cache holds
+    more than the trigger and more than K_min.  Equal budgets give R7.
 """
 from __future__ import annotations
 
@@ -288,6 +295,55 @@ def select_kept_chunked(scores, positions, K, prefill=0, recency_cap=128, chunk=
             break
     kept = set(range(P)) | set(range(n - R, n)) | set(best)
     return sorted(kept)
+
+
+def layer_recency(budgets, prefill, n, recency_cap=128):
+    """The recency window every layer keeps under per-layer budgets (R19)."""
+    k_min = min(budgets)
+    P = min(prefill, n)
+    return min(recency_window(k_min, recency_cap), max(0, k_min - P))
+
+
+def select_kept_layer(scores, K, prefill, R):
+    """One layer's ascending kept slot list of its own cache (R19): prefill,
+    the last R slots and the K - P - R best other slots (R8 order)."""
+    scores = np.asarray(scores, dtype=np.float64)
+    n = scores.shape[0]
+    P = min(prefill, n)
+    assert n >= P + R, "a layer holds the prefill and the recency window"
+    M = max(0, K - P - R)
+    candidates = list(range(P, n - R))
+
+    def rank(i):  # NaN last, higher score first, lower slot first
+        s = scores[i]
+        return (1, 0.0, i) if np.isnan(s) else (0, -s, i)
+
+    best = sorted(candidates, key=rank)[:M]
+    return sorted(set(range(P)) | set(range(n - R, n)) | set(best))
+
+
+def simulate_decode_layers(scores, length, chunk, budgets, trigger, prefill=0, recency_cap=128):
+    """Per-layer budgets (R19): every layer keeps its own cache of positions,
+    appends ``chunk`` tokens at a time and, whenever the largest cache holds
+    more than ``trigger`` tokens, evicts its own cache with its own budget.
+
+    Returns the events as [(per-layer positions before, after)] and the final
+    per-layer position lists.
+    """
+    caches = [[] for _ in budgets]
+    events = []
+    for start in range(0, length, chunk):
+        new = list(range(start, min(length, start + chunk)))
+        for c in caches:
+            c.extend(new)
+        n = max(len(c) for c in caches)
+        if n > trigger and n > min(budgets):        # some layer is over its budget
+            R = layer_recency(budgets, prefill, n, recency_cap)
+            before = [list(c) for c in caches]
+            caches = [[c[i] for i in select_kept_layer([scores[p] for p in c], K, prefill, R)]
+                      for c, K in zip(caches, budgets)]
+            events.append((before, [list(c) for c in caches]))
+    return events, caches
 
 
 # --------------------------------------------------------------------------

@@ -458,6 +458,98 @@ def test_chunked_select_structure_on_decode_histories():
             if kept_means and dropped_means:
                 assert min(kept_means) >= max(dropped_means) - 1e-6
 
+
+# ------------------------------------------ per-layer budgets (Sec. 5 future work)
+def test_layer_budgets_hand_example():
+    events_expected = {}
+    with open(os.path.join(GOLDEN, "layer_budgets_hand_example.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            head, *rest = line.split()
+            if head == "score":
+                score = [float(x) for x in rest]
+            elif head == "setup":
+                chunk, trigger, P, *budgets = (int(x) for x in rest)
+            elif head == "event":
+                events_expected[(int(rest[0]), int(rest[2]))] = [int(x) for x in rest[4:]]
+    events, final = O.simulate_decode_layers(score, len(score), chunk, budgets, trigger, prefill=P)
+    assert len(events) == 2
+    for (e, l), after in events_expected.items():
+        assert events[e][1][l] == after
+
+
+def test_equal_layer_budgets_are_the_token_rule():
+    rng = np.random.default_rng(31)
+    for trial in range(20):
+        L = 1000
+        s = rng.normal(size=L)
+        if trial % 4 == 0:
+            s[rng.integers(0, L, size=20)] = np.nan
+        K, P = int(rng.integers(20, 300)), int(rng.integers(0, 12))
+        chunk = int(rng.integers(1, 40))
+        trig = K + int(rng.integers(0, 30))
+        ev1, fin1 = O.simulate_decode(s, L, chunk, K, trig, prefill=P)
+        evl, finl = O.simulate_decode_layers(s, L, chunk, [K] * 3, trig, prefill=P)
+        assert [a for _, a in ev1] == [a[0] for _, a in evl] == [a[2] for _, a in evl]
+        assert finl == [fin1] * 3
+
+
+def _brute_layer(s, K, P, R):
+    n = len(s)
+    P = min(P, n)
+    M = max(0, K - P - R)
+    cand = list(range(P, n - R))
+    valid = [S for S in itertools.combinations(cand, min(M, len(cand)))
+             if all(_better(s, i, j) for i in S for j in cand if j not in S)]
+    assert len(valid) == 1
+    return sorted(set(range(P)) | set(range(n - R, n)) | set(valid[0]))
+
+
+def test_layer_selection_equals_brute_force_on_tiny_inputs():
+    rng = np.random.default_rng(32)
+    for trial in range(300):
+        n = int(rng.integers(1, 11))
+        P = int(rng.integers(0, 3))
+        R = int(rng.integers(0, max(1, n - min(P, n) + 1)))
+        K = int(rng.integers(1, 12))
+        s = rng.integers(-2, 3, size=n).astype(np.float64)
+        if trial % 5 == 0:
+            s[rng.integers(0, n)] = np.nan
+        assert O.select_kept_layer(s, K, P, R) == _brute_layer(list(s), K, P, R)
+
+
+def test_layer_caches_stay_nested_on_decode_histories():
+    """With one recency window and common events, a layer's cache after every
+    event is its own budget's selection from any larger layer's cache, so the
+    caches are nested; each keeps the prefill, the shared window and exactly
+    min(size, K_l) tokens."""
+    rng = np.random.default_rng(33)
+    for trial in range(12):
+        L = 1200
+        s = rng.normal(size=L)
+        n_layers = int(rng.integers(2, 6))
+        budgets = [int(x) for x in rng.integers(40, 400, size=n_layers)]
+        P = int(rng.integers(0, 10))
+        chunk = int(rng.integers(1, 50))
+        trig = max(budgets) + int(rng.integers(0, 40))
+        events, final = O.simulate_decode_layers(s, L, chunk, budgets, trig, prefill=P)
+        assert len(events) >= 2
+        order = sorted(range(n_layers), key=lambda l: -budgets[l])
+        for before, after in events:
+            n = max(len(b) for b in before)
+            R = min(min(128, min(budgets) // 4), max(0, min(budgets) - min(P, n)))
+            for l in range(n_layers):
+                assert len(after[l]) == min(len(before[l]), budgets[l])
+                assert after[l][:P] == list(range(min(P, n)))
+                if R:
+                    assert after[l][-R:] == before[l][-R:] == before[order[0]][-R:]
+            for a, b in zip(order, order[1:]):
+                big, small = after[a], after[b]
+                assert set(small) <= set(big)
+                sel = O.select_kept_layer([s[p] for p in big], budgets[b], P, R)
+                assert [big[i] for i in sel] == small
+
 # ------------------------------------------- the other attention-free variants
 def test_hsvar_closed_forms():
     # a walk with constant step a in Band A and b in Band B: g-bar = a, b
