@@ -107,6 +107,19 @@ typedef struct {
                              * (summed in slot order), and whole chunks fill the candidate
                              * budget in rank order (NaN lowest, ties to the earlier chunk);
                              * the first chunk that does not fit keeps its lowest slots. */
+  int32_t layer_budgets;    /* 0: one budget per sequence (the paper's method).  1: one budget
+                             * per (sequence, layer), which the paper names as future work
+                             * (Sec. 5, after PyramidKV's per-layer allocation, Sec. 2): layer
+                             * l keeps its own cache of n_l slots and evicts it with its own
+                             * budget K_l at the sequence's events; every layer keeps the
+                             * prefill and one shared recency window R = min(recency_cap,
+                             * K_min/4) (shrunk to K_min - P), K_min the smallest budget.
+                             * Needs num_layers <= 64 and select_chunk <= 1.  In this mode
+                             * the per-entry budget, kept and length arrays of epikv_select,
+                             * epikv_compact and epikv_step gain a layer dimension (see
+                             * there), "n_cache" is the largest layer's length, and the new
+                             * K/V rows of an update go to slots n_l .. n_l+n_new-1 of each
+                             * layer. */
 } epikv_config;
 
 /* New hidden-state rows of one update call (Sec. 3.1: the per-layer hidden
@@ -141,8 +154,8 @@ typedef struct {
 typedef struct {
   unsigned long long tokens_scored;  /* new tokens accepted by score updates */
   unsigned long long evictions;      /* (sequence, event) pairs that evicted */
-  unsigned long long rows_moved;     /* kept tokens whose slot changed */
-  unsigned long long reserved;
+  unsigned long long rows_moved;     /* kept tokens whose slot changed (largest layer) */
+  unsigned long long layer_rows_moved; /* (layer, kept token) pairs whose slot changed */
 } epikv_stats;
 
 typedef struct epikv_ctx epikv_ctx;
@@ -186,6 +199,16 @@ epikv_status epikv_score_update(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_
  *   d_kept    device int32 [n_seq][kept_stride]: ascending kept slots,
  *             written only for entries that evict
  *   d_n_kept  device int32 [n_seq]: the cache length after the call
+ * With cfg.layer_budgets = 1: d_budget is [n_seq][num_layers] (K_l of each
+ * layer), an entry evicts if n_cache (its largest layer) exceeds the trigger
+ * (NULL: the largest K_l) and the smallest K_l; d_kept is
+ * [n_seq][num_layers][kept_stride], each layer's kept slots in its own slot
+ * numbering, and d_n_kept is [n_seq][num_layers]; kept_stride must be at
+ * least max(K_max, prefill).  A sequence's layer budgets must stay the same
+ * from one epikv_seq_reset to the next: the library keeps one ranking for
+ * all layers, which is exact because fixed budgets keep the layers' caches
+ * nested; a change that would break the nesting is reported as
+ * EPIKV_DEV_KEPT.
  * Ties between equal scores go to the lower slot, NaN ranks lowest.  The
  * call commits the eviction to the context's slot metadata (scores and
  * positions move with their tokens); the caller must apply epikv_compact
@@ -196,7 +219,8 @@ epikv_status epikv_select(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_id
 
 /* Move every layer's K and V rows of the entries that evicted in the
  * preceding epikv_select to their kept slots, in order, in place (App. H).
- * Rows before the first evicted slot are not touched. */
+ * Rows before the first evicted slot are not touched.  d_kept has the layout
+ * epikv_select wrote (per layer with cfg.layer_budgets = 1). */
 epikv_status epikv_compact(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
                            const int32_t* d_kept, int32_t kept_stride, const epikv_kv_view* kv,
                            cudaStream_t stream);
@@ -205,7 +229,9 @@ epikv_status epikv_compact(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_i
  * (evict entries with n_cache > trigger), epikv_select into the context's
  * own kept buffer and epikv_compact -- without any host synchronisation.
  *   d_n_cache_out [n_seq] device or NULL: each entry's cache length after
- *                 the step (a paged caller frees blocks past it). */
+ *                 the step (a paged caller frees blocks past it);
+ *                 [n_seq][num_layers], every layer's length, with
+ *                 cfg.layer_budgets = 1 (d_budget as in epikv_select). */
 epikv_status epikv_step(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
                         const int32_t* d_cu_new, int32_t max_new, const int32_t* d_budget,
                         const int32_t* d_trigger, const epikv_hidden_view* hidden,
@@ -220,6 +246,12 @@ epikv_status epikv_set_phase_events(epikv_ctx* ctx, const cudaEvent_t* events);
  * scores of kind `kind` of `seq`'s slots; at most `cap` entries copied. */
 epikv_status epikv_read_slots(epikv_ctx* ctx, int32_t seq, int32_t kind, float* h_score,
                               int32_t* h_pos, int32_t cap, int32_t* h_n);
+
+/* Debug/test read-back (synchronises), cfg.layer_budgets = 1 only: the
+ * length n_l of layer `layer` of `seq` and the positions its slots hold, at
+ * most `cap` of them. */
+epikv_status epikv_read_layer_slots(epikv_ctx* ctx, int32_t seq, int32_t layer, int32_t* h_pos,
+                                    int32_t cap, int32_t* h_n);
 
 /* Synchronise the last stream used and return the cumulative counters. */
 epikv_status epikv_get_stats(epikv_ctx* ctx, epikv_stats* out);

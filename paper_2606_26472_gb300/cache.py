@@ -67,3 +67,15 @@ class KVCache:
         off = slots % self.block_size
         flat = torch.as_tensor(blk * self.block_size + off, device=pool.device)
         return pool.reshape(self.L, -1, self.H, self.d).index_select(1, flat).permute(1, 0, 2, 3)
+
+    def write_layer_rows(self, kind, seq, layer, slots, rows, block_table_host=None):
+        """Store bf16 rows [n, H, d] into the given slots of one layer (per-layer
+        budgets give each layer its own slot numbering)."""
+        pool = self.k if kind == 0 else self.v
+        slots = np.asarray(slots, dtype=np.int64)
+        if self.layout == E.EPIKV_LAYOUT_CONTIGUOUS:
+            pool[layer, seq][torch.as_tensor(slots, device=pool.device)] = rows
+            return
+        bt = block_table_host if block_table_host is not None else self.block_table.cpu().numpy()
+        flat = bt[seq][slots // self.block_size] * self.block_size + slots % self.block_size
+        pool[layer].view(-1, self.H, self.d)[torch.as_tensor(flat, device=pool.device)] = rows

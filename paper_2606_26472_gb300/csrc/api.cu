@@ -43,6 +43,8 @@ bool valid_config(const epikv_config* c) {
   if (c->score_kinds < 1 || c->score_kinds > 63) return false;
   if (c->recency_cap < 0) return false;
   if (c->select_chunk < 0 || c->select_chunk > 65536) return false;
+  if (c->layer_budgets != 0 && c->layer_budgets != 1) return false;
+  if (c->layer_budgets && (c->num_layers > 64 || c->select_chunk > 1)) return false;
   if (c->num_layers < 1 || c->num_kv_heads < 1 || c->num_kv_heads > 32) return false;
   if (!is_pow2(c->head_dim) || c->head_dim < 8 || c->head_dim > 256) return false;
   if (c->num_kv_heads * c->head_dim / 8 > 256) return false;
@@ -70,6 +72,7 @@ Dims make_dims(const epikv_config* c) {
   d.kinds = c->score_kinds;
   d.recency_cap = c->recency_cap;
   d.select_chunk = c->select_chunk > 1 ? c->select_chunk : 1;
+  d.layer_budgets = c->layer_budgets;
   const bool bz = c->score_kinds & kBandKinds, lg = c->score_kinds & kKvKinds;
   d.D = bz ? c->hidden : 0;
   d.nA = bz ? c->n_band_a : 0;
@@ -105,8 +108,9 @@ size_t carve(const Dims& d, DevState* st, char* base) {
   st->err = (int32_t*)take(4);
   st->stats = (unsigned long long*)take(4 * 8);
   st->pos = (int32_t*)take(S * T * 4);
-  st->kept = (int32_t*)take(S * T * 4);
-  st->n_kept = (int32_t*)take(S * 4);
+  const size_t LB = d.layer_budgets ? (size_t)d.L : 1;  // kept lists and lengths per layer
+  st->kept = (int32_t*)take(S * LB * T * 4);
+  st->n_kept = (int32_t*)take(S * LB * 4);
   for (int k = 0; k < kNumKinds; ++k)
     if (d.kinds & (1 << k)) st->score[k] = (float*)take(S * T * 4);
   if (d.kinds & kBandKinds) {
@@ -122,6 +126,13 @@ size_t carve(const Dims& d, DevState* st, char* base) {
   for (int q = 0; q < 4; ++q)
     if (d.kinds & kv_kind(q)) st->u_ring[q] = (float*)take(S * (size_t)d.G * 4);
   if (d.select_chunk > 1) st->ckey = (uint32_t*)take(S * T * 4);
+  if (d.layer_budgets) {
+    st->n_layer = (int32_t*)take(S * d.L * 4);
+    st->lfirst = (int32_t*)take(S * d.L * 4);
+    st->lmask = (unsigned long long*)take(S * T * 8);
+    st->lmask_new = (unsigned long long*)take(S * T * 8);
+    st->mkept = (int32_t*)take(S * T * 4);
+  }
   return align_up(off, 256);
 }
 
@@ -313,6 +324,38 @@ epikv_status epikv_read_slots(epikv_ctx* ctx, int32_t seq, int32_t kind, float* 
   if (e == cudaSuccess && m > 0 && h_score)
     e = cudaMemcpy(h_score, ctx->st.score[kind_index(kind)] + (size_t)seq * ctx->dm.T, (size_t)m * 4,
                    cudaMemcpyDeviceToHost);
+  return cuda_status(e);
+}
+
+epikv_status epikv_read_layer_slots(epikv_ctx* ctx, int32_t seq, int32_t layer, int32_t* h_pos, int32_t cap,
+                                    int32_t* h_n) {
+  if (!ctx || !ctx->dm.layer_budgets || seq < 0 || seq >= ctx->dm.S || layer < 0 || layer >= ctx->dm.L || cap < 0 ||
+      !h_n)
+    return EPIKV_EINVAL;
+  cudaError_t e = cudaStreamSynchronize(ctx->last_stream);
+  int32_t n = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&n, ctx->st.n_cache + seq, 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return EPIKV_ECUDA;
+  int32_t* pos = (int32_t*)malloc((size_t)(n > 0 ? n : 1) * 4);
+  unsigned long long* mask = (unsigned long long*)malloc((size_t)(n > 0 ? n : 1) * 8);
+  if (!pos || !mask) {
+    free(pos);
+    free(mask);
+    return EPIKV_EINVAL;
+  }
+  const size_t base = (size_t)seq * ctx->dm.T;
+  if (n > 0) e = cudaMemcpy(pos, ctx->st.pos + base, (size_t)n * 4, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && n > 0) e = cudaMemcpy(mask, ctx->st.lmask + base, (size_t)n * 8, cudaMemcpyDeviceToHost);
+  int32_t nl = 0;
+  if (e == cudaSuccess)
+    for (int i = 0; i < n; ++i)
+      if ((mask[i] >> layer) & 1ull) {
+        if (h_pos && nl < cap) h_pos[nl] = pos[i];
+        ++nl;
+      }
+  free(pos);
+  free(mask);
+  *h_n = nl;
   return cuda_status(e);
 }
 

@@ -54,11 +54,17 @@ struct DevState {
   int32_t* kept;           // [S][T] kept lists of epikv_step
   int32_t* n_kept;         // [S]
   uint32_t* ckey;          // [S][T] chunk-level selection: each candidate slot's chunk key (C > 1 only)
+  // per-layer budgets only (null otherwise)
+  int32_t* n_layer;        // [S][L] slots held by each layer
+  int32_t* lfirst;         // [S][L] first slot of each layer moved by the last selection
+  unsigned long long* lmask;      // [S][T] bit l: layer l holds the token of this slot
+  unsigned long long* lmask_new;  // [S][T] the select kernel's new masks (scratch)
+  int32_t* mkept;          // [S][T] the select kernel's kept slots of the largest layer (scratch)
 };
 
 struct Dims {
   int S, T, max_new, L, H, d, D, nA, nB, G;
-  int z_window, lag, lag_window, recency_cap, kinds, select_chunk;
+  int z_window, lag, lag_window, recency_cap, kinds, select_chunk, layer_budgets;
   float z_eps, lag_eps;
 };
 

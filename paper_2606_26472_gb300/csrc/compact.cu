@@ -13,6 +13,9 @@
 // increasing i, so a load (slot kept[i] >= i) never reads a slot that an
 // earlier store has written, and a later store to a slot some earlier batch
 // still had to read is issued only after that batch's loads completed.
+//
+// Under per-layer budgets (kLayers) each (sequence, layer) has its own kept
+// list, first moved slot and length; the streams and the copy are unchanged.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -52,6 +55,7 @@ struct Cursor {
   int b, seq, layer, kvk, hg;
 };
 
+template <bool kLayers>
 __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev kv,
                                                      const int32_t* __restrict__ seq_ids, int n_seq,
                                                      const int32_t* __restrict__ kept, int kept_stride) {
@@ -118,8 +122,13 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       c.hg = rem % hs;
       c.b = list[e];
       c.seq = seq_ids[c.b];
-      c.i = st.first_changed[c.seq];
-      c.end = st.n_cache[c.seq];
+      if (kLayers) {
+        c.i = st.lfirst[c.seq * dm.L + c.layer];
+        c.end = st.n_layer[c.seq * dm.L + c.layer];
+      } else {
+        c.i = st.first_changed[c.seq];
+        c.end = st.n_cache[c.seq];
+      }
       if (c.i < c.end) return;
       c.u += G;
     }
@@ -135,7 +144,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   auto prefetch = [&](const Cursor& c, int (&pk)[kMaxRowsPerLane]) {
     if (c.u >= units) return;
     const int nrows = min(rpb, c.end - c.i);
-    const int32_t* kl = kept + (size_t)c.b * kept_stride + c.i;
+    const int32_t* kl = kept + (kLayers ? (size_t)c.b * dm.L + c.layer : (size_t)c.b) * kept_stride + c.i;
 #pragma unroll
     for (int j = 0; j < kMaxRowsPerLane; ++j) {
       const int r = lane + 32 * j;
@@ -252,11 +261,14 @@ static size_t compact_smem(int n_seq) {
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm) {
   (void)device;
-  cudaError_t e = cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(compact_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)compact_smem(4096));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(compact_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)compact_smem(4096));
   if (e != cudaSuccess) return e;
   int n = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel, 32, compact_smem(64));
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel<false>, 32, compact_smem(64));
   if (e != cudaSuccess) return e;
   g_ctas_per_sm = n > 0 ? n : 1;
   if (EPIKV_COMPACT_CTAS_PER_SM > 0 && EPIKV_COMPACT_CTAS_PER_SM < g_ctas_per_sm) g_ctas_per_sm = EPIKV_COMPACT_CTAS_PER_SM;
@@ -268,7 +280,10 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
                            const int32_t* kept, int kept_stride, const KvDev& kv, int ctas,
                            cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
-  compact_kernel<<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  if (dm.layer_budgets)
+    compact_kernel<true><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  else
+    compact_kernel<false><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
   ++*launches;
   return cudaGetLastError();
 }

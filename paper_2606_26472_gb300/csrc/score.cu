@@ -229,7 +229,8 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
   const int h = tid / LH, q = tid % LH;
   const bool active = h < dm.H;
   const int hd = dm.H * dm.d;
-  const int nc0 = st.n_cache[seq];
+  // the new rows' first slot: this layer's own length under per-layer budgets
+  const int nc0 = dm.layer_budgets ? st.n_layer[seq * dm.L + layer] : st.n_cache[seq];
   const int p0 = st.n_seen[seq];
   if (nc0 + n_new > dm.T) {
     if (tid == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
@@ -396,6 +397,8 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
     for (int i = i_lo + warp; i < i_hi; i += kFinThreads / 32) {
       const int pos = p0 + i;
       if (lane == 0) st.pos[(size_t)seq * dm.T + nc0 + i] = pos;
+      if (lane == 0 && dm.layer_budgets)  // a new token is in every layer
+        st.lmask[(size_t)seq * dm.T + nc0 + i] = dm.L == 64 ? ~0ull : (1ull << dm.L) - 1ull;
     }
     if (dm.kinds & kBandKinds) {
       // every g value the tile's windows reach, all band layers, one round of loads
@@ -511,6 +514,8 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
       if (fits) {
         st.n_cache[seq] = nc0 + n_new;
         st.n_seen[seq] = p0 + n_new;
+        if (dm.layer_budgets)
+          for (int l = 0; l < dm.L; ++l) st.n_layer[seq * dm.L + l] += n_new;
         if ((dm.kinds & kBandKinds) && n_new > 0) st.hp_parity[seq] ^= 1;
         atomicAdd(&st.stats[0], (unsigned long long)n_new);
       }

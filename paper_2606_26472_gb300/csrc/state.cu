@@ -21,6 +21,11 @@ __global__ void reset_seq_kernel(DevState st, Dims dm, int seq, int prefill, int
     st.ticket[seq] = 0u;
     st.n_kept[seq] = 0;
   }
+  if (dm.layer_budgets)
+    for (int l = threadIdx.x; l < dm.L; l += blockDim.x) {
+      st.n_layer[seq * dm.L + l] = 0;
+      st.lfirst[seq * dm.L + l] = 0;
+    }
 }
 
 cudaError_t launch_init_state(const DevState& st, const Dims& dm, cudaStream_t stream) {

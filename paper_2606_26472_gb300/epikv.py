@@ -24,7 +24,7 @@ class epikv_config(C.Structure):
                 ("hidden", C.c_int32), ("n_band_a", C.c_int32), ("n_band_b", C.c_int32),
                 ("z_window", C.c_int32), ("z_eps", C.c_float), ("lag", C.c_int32), ("lag_eps", C.c_float),
                 ("lag_window", C.c_int32), ("recency_cap", C.c_int32), ("score_kinds", C.c_int32),
-                ("select_chunk", C.c_int32)]
+                ("select_chunk", C.c_int32), ("layer_budgets", C.c_int32)]
 
 
 class epikv_hidden_view(C.Structure):
@@ -40,7 +40,7 @@ class epikv_kv_view(C.Structure):
 
 class epikv_stats(C.Structure):
     _fields_ = [("tokens_scored", C.c_ulonglong), ("evictions", C.c_ulonglong), ("rows_moved", C.c_ulonglong),
-                ("reserved", C.c_ulonglong)]
+                ("layer_rows_moved", C.c_ulonglong)]
 
 
 _P = C.c_void_p
@@ -57,6 +57,7 @@ _SIGS = {
                              C.POINTER(epikv_kv_view), _P, _P]),
     "epikv_set_phase_events": (C.c_int, [_P, _P]),
     "epikv_read_slots": (C.c_int, [_P, _I, _I, _P, _P, _I, C.POINTER(_I)]),
+    "epikv_read_layer_slots": (C.c_int, [_P, _I, _I, _P, _I, C.POINTER(_I)]),
     "epikv_get_stats": (C.c_int, [_P, C.POINTER(epikv_stats)]),
     "epikv_get_error": (C.c_int, [_P, C.POINTER(_I)]),
     "epikv_lagkv_score_noalloc": (C.c_int, [C.POINTER(epikv_kv_view), _I, _I, _I, _I, _I, _I, C.c_float, _I,
@@ -115,10 +116,10 @@ def _stream(s):
 
 def make_config(*, max_seqs, max_cache_tokens, max_new_tokens, num_layers=32, num_kv_heads=8, head_dim=128,
                 hidden=4096, n_band_a=7, n_band_b=8, z_window=64, z_eps=1e-6, lag=16, lag_eps=1e-6,
-                lag_window=64, recency_cap=128, score_kinds=EPIKV_SCORE_BANDZ, select_chunk=1):
+                lag_window=64, recency_cap=128, score_kinds=EPIKV_SCORE_BANDZ, select_chunk=1, layer_budgets=0):
     return epikv_config(max_seqs, max_cache_tokens, max_new_tokens, num_layers, num_kv_heads, head_dim, hidden,
                         n_band_a, n_band_b, z_window, z_eps, lag, lag_eps, lag_window, recency_cap, score_kinds,
-                        select_chunk)
+                        select_chunk, layer_budgets)
 
 
 def hidden_view(band_rows, row_stride):
@@ -194,10 +195,20 @@ def epikv_read_slots(ctx, seq, kind, cap):
     return list(pos[:m]), list(score[:m]), n.value
 
 
+def epikv_read_layer_slots(ctx, seq, layer, cap):
+    """Synchronising read-back under per-layer budgets: (positions of the
+    layer's slots as a list, the layer's length)."""
+    n = C.c_int32()
+    pos = (C.c_int32 * max(cap, 1))()
+    _check(load().epikv_read_layer_slots(ctx, seq, layer, pos, cap, C.byref(n)), "epikv_read_layer_slots")
+    return list(pos[:min(n.value, cap)]), n.value
+
+
 def epikv_get_stats(ctx):
     s = epikv_stats()
     _check(load().epikv_get_stats(ctx, C.byref(s)), "epikv_get_stats")
-    return {"tokens_scored": s.tokens_scored, "evictions": s.evictions, "rows_moved": s.rows_moved}
+    return {"tokens_scored": s.tokens_scored, "evictions": s.evictions, "rows_moved": s.rows_moved,
+            "layer_rows_moved": s.layer_rows_moved}
 
 
 def epikv_get_error(ctx):

@@ -72,7 +72,7 @@ class Session:
 
     def __init__(self, model, *, n_seq, kinds, layout, max_tokens, max_new, prefill, policies,
                  z_window=64, lag=16, lag_window=64, recency_cap=128, block_size=16, shuffle_blocks=True,
-                 select_chunk=1, device="cuda"):
+                 select_chunk=1, layer_budgets=0, device="cuda"):
         self.m = model
         self.n_seq = n_seq
         self.kinds = kinds
@@ -80,13 +80,16 @@ class Session:
         self.policies = list(policies)
         self.recency_cap = recency_cap
         self.select_chunk = select_chunk
+        self.layer_budgets = layer_budgets
+        self.L = model.num_layers
         self.max_new = max_new
         self.dt = DeviceTrace(model, device)
         self.cfg = E.make_config(max_seqs=n_seq, max_cache_tokens=max_tokens, max_new_tokens=max_new,
                                  num_layers=model.num_layers, num_kv_heads=model.num_kv_heads,
                                  head_dim=model.head_dim, hidden=model.hidden, n_band_a=len(model.band_a),
                                  n_band_b=len(model.band_b), z_window=z_window, lag=lag, lag_window=lag_window,
-                                 recency_cap=recency_cap, score_kinds=kinds, select_chunk=select_chunk)
+                                 recency_cap=recency_cap, score_kinds=kinds, select_chunk=select_chunk,
+                                 layer_budgets=layer_budgets)
         nbytes = E.epikv_workspace_bytes(self.cfg)
         assert nbytes > 0
         self.ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
@@ -110,8 +113,14 @@ class Session:
             if kinds & BAND_KINDS else None
         self.n_cache = [0] * n_seq
         self.n_seen = [0] * n_seq
-        self.kept = torch.empty((n_seq, max_tokens), dtype=torch.int32, device=device)
-        self.n_kept = torch.empty((n_seq,), dtype=torch.int32, device=device)
+        lay = (self.L,) if layer_budgets else ()
+        self.kept = torch.empty((n_seq,) + lay + (max_tokens,), dtype=torch.int32, device=device)
+        self.n_kept = torch.empty((n_seq,) + lay, dtype=torch.int32, device=device)
+        # per-layer budgets: each layer's length, and a one-sequence staging
+        # cache the new rows are generated into before each layer's copy
+        self.n_layer = [[0] * self.L for _ in range(n_seq)]
+        self.stage = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, model.num_layers, model.num_kv_heads, model.head_dim,
+                             max_seqs=1, max_tokens=max_new, device=device) if layer_budgets else None
 
     # ---------------------------------------------------------------- inputs
     def append(self, entries):
@@ -120,8 +129,17 @@ class Session:
         cu = [0]
         for b, n in entries:
             assert self.n_cache[b] + n <= self.cache.T
-            self.dt.kv(b, self.n_seen[b], n, self.n_cache[b], self.cache.k, self.cache.v,
-                       **self.cache.synth_kwargs())
+            if self.layer_budgets:
+                kw = self.stage.synth_kwargs()
+                kw["stride_seq"] = 0
+                self.dt.kv(b, self.n_seen[b], n, 0, self.stage.k, self.stage.v, **kw)
+                for l in range(self.L):
+                    slots = np.arange(self.n_layer[b][l], self.n_layer[b][l] + n)
+                    for kind, pool in ((0, self.stage.k), (1, self.stage.v)):
+                        self.cache.write_layer_rows(kind, b, l, slots, pool[l, 0, :n], self.bt_host)
+            else:
+                self.dt.kv(b, self.n_seen[b], n, self.n_cache[b], self.cache.k, self.cache.v,
+                           **self.cache.synth_kwargs())
             if self.hid is not None:
                 for i, layer in enumerate(self.m.band_layers):
                     out = self.hid[i, cu[-1]:cu[-1] + n]
@@ -141,6 +159,7 @@ class Session:
         for b, n in entries:
             self.n_cache[b] += n
             self.n_seen[b] += n
+            self.n_layer[b] = [x + n for x in self.n_layer[b]]
         self._keep_alive = (seq_ids, cu_new)
 
     def step(self, entries, budgets, triggers):
@@ -149,12 +168,16 @@ class Session:
         n = len(entries)
         bud = torch.tensor(budgets, dtype=torch.int32, device=self.ws.device)
         trig = torch.tensor(triggers, dtype=torch.int32, device=self.ws.device)
-        out = torch.empty(n, dtype=torch.int32, device=self.ws.device)
+        out = torch.empty((n, self.L) if self.layer_budgets else (n,), dtype=torch.int32, device=self.ws.device)
         E.epikv_step(self.ctx, n, seq_ids, cu_new, mx, bud, trig, hv, self.kv, out)
         lens = out.cpu().numpy()
         for i, (b, k) in enumerate(entries):
             self.n_seen[b] += k
-            self.n_cache[b] = int(lens[i])
+            if self.layer_budgets:
+                self.n_layer[b] = [int(x) for x in lens[i]]
+                self.n_cache[b] = max(self.n_layer[b])
+            else:
+                self.n_cache[b] = int(lens[i])
 
     def read(self, b, kind):
         pos, sc, n = E.epikv_read_slots(self.ctx, b, kind, self.cache.T)
@@ -165,12 +188,19 @@ class Session:
         seq_ids = torch.tensor(seqs, dtype=torch.int32, device=self.ws.device)
         bud = torch.tensor(budgets, dtype=torch.int32, device=self.ws.device)
         trig = None if triggers is None else torch.tensor(triggers, dtype=torch.int32, device=self.ws.device)
-        E.epikv_select(self.ctx, len(seqs), seq_ids, bud, trig, self.kept, self.kept.shape[1], self.n_kept)
+        E.epikv_select(self.ctx, len(seqs), seq_ids, bud, trig, self.kept, self.kept.shape[-1], self.n_kept)
         torch.cuda.synchronize()
         nk = self.n_kept[:len(seqs)].cpu().numpy()
         kept = self.kept[:len(seqs)].cpu().numpy()
         self._sel = (seq_ids,)
         out = {}
+        if self.layer_budgets:   # {b: per-layer kept lists} of the entries where some layer evicted
+            for i, b in enumerate(seqs):
+                if any(nk[i, l] < self.n_layer[b][l] for l in range(self.L)):
+                    out[b] = [kept[i, l, :nk[i, l]].astype(np.int64) for l in range(self.L)]
+                self.n_layer[b] = [int(x) for x in nk[i]]
+                self.n_cache[b] = max(self.n_layer[b])
+            return out
         for i, b in enumerate(seqs):
             if nk[i] < self.n_cache[b]:
                 out[b] = kept[i, :nk[i]].astype(np.int64)
@@ -179,7 +209,17 @@ class Session:
 
     def compact(self, seqs):
         seq_ids = self._sel[0]
-        E.epikv_compact(self.ctx, len(seqs), seq_ids, self.kept, self.kept.shape[1], self.kv)
+        E.epikv_compact(self.ctx, len(seqs), seq_ids, self.kept, self.kept.shape[-1], self.kv)
+
+    def read_layer(self, b, layer):
+        pos, n = E.epikv_read_layer_slots(self.ctx, b, layer, self.cache.T)
+        assert n == self.n_layer[b][layer], (b, layer, n, self.n_layer[b][layer])
+        return np.array(pos, dtype=np.int64)
+
+    def layer_rows_u16(self, b, layer, slots):
+        k = as_u16(self.cache.rows(0, b, slots, self.bt_host)[:, layer])
+        v = as_u16(self.cache.rows(1, b, slots, self.bt_host)[:, layer])
+        return k, v
 
     def error(self):
         return E.epikv_get_error(self.ctx)

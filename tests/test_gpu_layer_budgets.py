@@ -1,0 +1,190 @@
+"""Per-layer budgets on the GPU (the per-layer budgets the paper names as
+future work, Sec. 5).  The oracle evicts every layer's cache on its own; the
+GPU path keeps the union of the layers with a mask per slot and one ranking.
+Checked: every layer's positions after every event equal the oracle's
+replay on the GPU's own scores, every layer's compacted K/V rows are the
+generator's rows of those positions, equal budgets give the token-level
+path bit for bit, and the one-call step equals the split calls."""
+import numpy as np
+import pytest
+
+from oracle import epikv_oracle as O
+from paper_2606_26472_gb300 import epikv as E
+from synth import gen, workloads as W
+
+from .harness import OracleTrace, Session, assert_scores_close
+
+pytestmark = pytest.mark.gpu
+
+BANDZ, LAGKV = E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV
+
+
+class LayerReplay:
+    """The oracle's per-layer caches of one sequence, replayed on the GPU's
+    frozen scores with the same schedule."""
+
+    def __init__(self, n_layers, budgets, prefill, trigger):
+        self.caches = [[] for _ in range(n_layers)]
+        self.budgets, self.prefill, self.trigger = list(budgets), prefill, trigger
+        self.score = {}
+
+    def append(self, positions, scores):
+        for p, s in zip(positions, scores):
+            self.score[int(p)] = float(s)
+        for c in self.caches:
+            c.extend(int(p) for p in positions)
+
+    def event(self):
+        n = max(len(c) for c in self.caches)
+        if not (n > self.trigger and n > min(self.budgets)):
+            return False
+        R = O.layer_recency(self.budgets, self.prefill, n)
+        self.caches = [[c[i] for i in O.select_kept_layer([self.score[p] for p in c], K, self.prefill, R)]
+                       for c, K in zip(self.caches, self.budgets)]
+        return True
+
+
+def _check_layer_bytes(sess, b, layer, positions):
+    slots = np.arange(len(positions))
+    k, v = sess.layer_rows_u16(b, layer, slots)
+    pos = np.asarray(positions)
+    sp = gen.spike_flags(sess.m, b, int(pos.max()) + 1)
+    np.testing.assert_array_equal(k, gen.kv_rows(sess.m, sess.dt.tabs, b, 0, pos, sp)[:, layer])
+    np.testing.assert_array_equal(v, gen.kv_rows(sess.m, sess.dt.tabs, b, 1, pos, sp)[:, layer])
+
+
+CASES = [
+    # layout, kinds, prefill, per-sequence layer budgets (small model: 4 layers), new-token pattern
+    ("contig_bandz", E.EPIKV_LAYOUT_CONTIGUOUS, BANDZ, (0, 5, 0),
+     ((100, 80, 60, 40), (64, 64, 64, 64), (40, 90, 70, 120)), (7, 1, 33)),
+    ("paged_lag", E.EPIKV_LAYOUT_PAGED, LAGKV, (0, 3, 20),
+     ((48, 96, 72, 120), (130, 30, 30, 130), (60, 61, 62, 63)), (16, 5, 40)),
+    ("paged_both", E.EPIKV_LAYOUT_PAGED, BANDZ | LAGKV, (3, 0, 0),
+     ((80, 50, 110, 20), (33, 66, 99, 132), (90, 90, 45, 45)), (1, 9, 64)),
+]
+
+
+@pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks", CASES, ids=[c[0] for c in CASES])
+def test_layer_budget_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chunks):
+    model = W.small_model(2000 + len(name))
+    n_seq, L = 3, model.num_layers
+    lengths = (301, 260, 333)
+    slack = 10
+    policies = [BANDZ if (kinds & BANDZ and (b % 2 == 0 or kinds == BANDZ)) else LAGKV for b in range(n_seq)]
+    max_new = max(chunks)
+    T_cap = max(max(k) for k in budgets) + slack + max_new + 1
+    sess = Session(model, n_seq=n_seq, kinds=kinds, layout=layout, max_tokens=T_cap, max_new=max_new,
+                   prefill=prefill, policies=policies, layer_budgets=1)
+    refs = [OracleTrace(model, sess.dt.tabs, b, lengths[b], kinds) for b in range(n_seq)]
+    triggers = [max(budgets[b]) + slack for b in range(n_seq)]
+    replay = [LayerReplay(L, budgets[b], prefill[b], triggers[b]) for b in range(n_seq)]
+    events, step = 0, 0
+    while any(sess.n_seen[b] < lengths[b] for b in range(n_seq)):
+        entries = []
+        for b in range(n_seq):
+            n = min(chunks[(b + step) % len(chunks)], lengths[b] - sess.n_seen[b])
+            if n > 0:
+                entries.append((b, n))
+        step += 1
+        before = {b: sess.n_cache[b] for b, _ in entries}
+        sess.score_update(entries)
+        for b, n in entries:
+            pos, sc = sess.read(b, policies[b])
+            new = slice(before[b], before[b] + n)
+            np.testing.assert_array_equal(pos[new], np.arange(sess.n_seen[b] - n, sess.n_seen[b]))
+            assert_scores_close(sc[new], refs[b].scores[policies[b]][pos[new]], f"{name} seq {b}")
+            replay[b].append(pos[new], sc[new])
+        seqs = [b for b, _ in entries]
+        kept = sess.select(seqs, [list(budgets[b]) for b in seqs], [triggers[b] for b in seqs])
+        sess.compact(seqs)
+        for b in seqs:
+            fired = replay[b].event()
+            assert (b in kept) <= fired
+            events += fired
+            for l in range(L):
+                got = sess.read_layer(b, l)
+                assert list(got) == replay[b].caches[l], f"{name} seq {b} layer {l} step {step}"
+            if fired and step % 3 == 0:
+                for l in range(L):
+                    _check_layer_bytes(sess, b, l, replay[b].caches[l])
+    assert events >= 6
+    for b in range(n_seq):
+        for l in range(L):
+            _check_layer_bytes(sess, b, l, replay[b].caches[l])
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
+def test_equal_layer_budgets_are_the_token_path_bit_for_bit(gpu_lib):
+    model = W.small_model(63)
+    kw = dict(n_seq=2, kinds=BANDZ | LAGKV, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=180, max_new=20,
+              prefill=(3, 0), policies=(BANDZ, LAGKV))
+    a, b = Session(model, layer_budgets=1, **kw), Session(model, **kw)
+    K, slack = (100, 70), 12
+    for step in range(25):
+        entries = [(s, (7, 20, 3)[(s + step) % 3]) for s in range(2)]
+        a.score_update(entries)
+        b.score_update(entries)
+        ka = a.select([0, 1], [[K[s]] * model.num_layers for s in range(2)], [K[s] + slack for s in range(2)])
+        kb = b.select([0, 1], list(K), [K[s] + slack for s in range(2)])
+        a.compact([0, 1])
+        b.compact([0, 1])
+        assert set(ka) == set(kb)
+        for s in ka:
+            for l in range(model.num_layers):
+                np.testing.assert_array_equal(ka[s][l], kb[s])
+        for s in range(2):
+            assert a.n_cache[s] == b.n_cache[s] and a.n_layer[s] == [b.n_cache[s]] * model.num_layers
+            for kind in (BANDZ, LAGKV):
+                pa, sa = a.read(s, kind)
+                pb, sb = b.read(s, kind)
+                np.testing.assert_array_equal(pa, pb)
+                np.testing.assert_array_equal(sa.view(np.uint32), sb.view(np.uint32))
+    for s in range(2):
+        n = a.n_cache[s]
+        np.testing.assert_array_equal(np.stack(a.cache_rows_u16(s, np.arange(n))),
+                                      np.stack(b.cache_rows_u16(s, np.arange(n))))
+    assert E.epikv_get_stats(a.ctx)["layer_rows_moved"] == E.epikv_get_stats(b.ctx)["layer_rows_moved"] > 0
+    assert a.error() == b.error() == (E.EPIKV_OK, 0)
+    a.close()
+    b.close()
+
+
+def test_layer_budget_step_equals_split_calls(gpu_lib):
+    model = W.small_model(64)
+    kw = dict(n_seq=3, kinds=LAGKV, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=220, max_new=24,
+              prefill=(0, 4, 1), policies=(LAGKV,) * 3, layer_budgets=1)
+    a, b = Session(model, **kw), Session(model, **kw)
+    budgets = [[120, 90, 60, 30], [50, 50, 100, 100], [64, 128, 96, 32]]
+    triggers = [max(k) + 9 for k in budgets]
+    for step in range(30):
+        entries = [(s, (24, 2, 11)[(s + step) % 3]) for s in range(3)]
+        a.step(entries, budgets, triggers)
+        b.score_update(entries)
+        b.select([0, 1, 2], budgets, triggers)
+        b.compact([0, 1, 2])
+        for s in range(3):
+            assert a.n_layer[s] == b.n_layer[s]
+            for l in range(model.num_layers):
+                np.testing.assert_array_equal(a.read_layer(s, l), b.read_layer(s, l))
+    for s in range(3):
+        for l in range(model.num_layers):
+            n = a.n_layer[s][l]
+            np.testing.assert_array_equal(np.stack(a.layer_rows_u16(s, l, np.arange(n))),
+                                          np.stack(b.layer_rows_u16(s, l, np.arange(n))))
+    assert a.error() == b.error() == (E.EPIKV_OK, 0)
+    a.close()
+    b.close()
+
+
+def test_a_bad_layer_budget_is_reported_and_nothing_moves(gpu_lib):
+    model = W.small_model(65)
+    sess = Session(model, n_seq=1, kinds=BANDZ, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=80, max_new=80,
+                   prefill=(0,), policies=(BANDZ,), layer_budgets=1)
+    sess.score_update([(0, 80)])
+    before = [sess.read_layer(0, l) for l in range(model.num_layers)]
+    assert sess.select([0], [[40, 0, 40, 40]]) == {}
+    assert sess.error() == (E.EPIKV_EDEVICE, E.EPIKV_DEV_BUDGET)
+    for l in range(model.num_layers):
+        np.testing.assert_array_equal(sess.read_layer(0, l), before[l])
+    sess.close()
