@@ -57,7 +57,7 @@ def parse():
     p.add_argument("--chunk", type=int, default=128)
     # the band-z kernels' workload: the 2,048-token single-sequence case, one
     # fresh sequence per step (reported for the per-kernel rooflines)
-    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken"])
+    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken", "layers32k"])
     # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
     # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
     p.add_argument("--kinds", type=int, default=2)
@@ -653,6 +653,142 @@ def run_pertoken(args):
     print(json.dumps(line), flush=True)
 
 
+def run_layers32k(args):
+    """Per-layer budgets on the 32 x 32k Lag-KV paged workload: layer l of
+    every sequence keeps its own budget K_l (a pyramid from 1.5 K at layer 0
+    to 0.5 K at the last layer, mean K) and every step evicts every layer
+    (trigger K_max + C - 1).  One step = C new tokens per sequence: scoring,
+    the per-layer selection and the per-layer compaction (epikv_step).  Each
+    step's new K/V rows go to every layer's own next slots, which depend on
+    the previous step, so they are written between steps, untimed (in a
+    decode loop the model's forward writes them); the time is the sum of the
+    steps' device times (CUDA events on the launching stream)."""
+    import torch
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    from paper_2606_26472_gb300.cache import KVCache
+    from synth import gen, workloads as W
+    from synth.device import DeviceTrace
+
+    rank, local_rank, world = dist_env()
+    assert world == 1, "the per-layer budget workload is a single-GPU measurement"
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+    wl = W.config(3)
+    m = wl.model
+    Bn, K, C = args.sequences, args.budget, args.chunk
+    L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
+    bs = wl.block_size
+    budgets = W.pyramid_budgets(K, L)
+    K_max = max(budgets)
+    T_cap = K_max + C
+    assert T_cap % bs == 0
+    mb = T_cap // bs
+    n_blocks = Bn * mb
+    perm = gen.block_permutation(m.seed, n_blocks).reshape(Bn, mb)
+    cache = KVCache(E.EPIKV_LAYOUT_PAGED, L, H, d, max_seqs=Bn, max_tokens=T_cap, block_size=bs,
+                    num_blocks=n_blocks, block_table=perm, device=dev)
+    view = cache.view()
+    stage = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, L, H, d, max_seqs=Bn, max_tokens=C, device=dev)
+    dt = DeviceTrace(m, dev)
+    stream = torch.cuda.current_stream()
+    cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T_cap, max_new_tokens=C, num_layers=L, num_kv_heads=H,
+                        head_dim=d, lag=wl.lag, lag_window=wl.lag_window, recency_cap=wl.recency_cap,
+                        score_kinds=E.EPIKV_SCORE_LAGKV, layer_budgets=1)
+    ws = torch.empty(E.epikv_workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws.numel())
+    for b in range(Bn):
+        E.epikv_seq_reset(ctx, b, 0, E.EPIKV_SCORE_LAGKV)
+    seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
+    cu_new = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * C).contiguous()
+    # the first K_fill tokens of every trace, in every layer, scored C at a time (no eviction yet)
+    K_fill = K_max // C * C
+    for b in range(Bn):
+        dt.kv(b, 0, K_fill, 0, cache.k, cache.v, **cache.synth_kwargs())
+    for _ in range(K_fill // C):
+        E.epikv_score_update(ctx, Bn, seq_ids, cu_new, C, None, view)
+    budget = torch.tensor([list(budgets)] * Bn, dtype=torch.int32, device=dev)
+    trigger = torch.full((Bn,), K_max + C - 1, dtype=torch.int32, device=dev)
+    n_out = torch.empty((Bn, L), dtype=torch.int32, device=dev)
+    n_layer = np.full((Bn, L), K_fill, dtype=np.int64)
+    rows = np.arange(Bn)[:, None]
+
+    def write_new(pos0):   # step's new rows into every layer's next C slots
+        for b in range(Bn):
+            dt.kv(b, pos0, C, 0, stage.k, stage.v, **stage.synth_kwargs())
+        for l in range(L):
+            slots = n_layer[:, l:l + 1] + np.arange(C)
+            flat = perm[rows, slots // bs] * bs + slots % bs
+            idx = torch.as_tensor(flat.reshape(-1), device=dev)
+            cache.k[l].view(-1, H, d)[idx] = stage.k[l].reshape(-1, H, d)
+            cache.v[l].view(-1, H, d)[idx] = stage.v[l].reshape(-1, H, d)
+
+    n_steps = args.warmup + args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_steps)]
+    phase = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_steps)]
+    for e in (x for p in phase for x in p):
+        e.record(stream)   # materialise the handles
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        gpu_id = str(local_rank)
+    clocks = None
+    stats0 = None
+    for st in range(n_steps):
+        if st == args.warmup:
+            torch.cuda.synchronize()
+            stats0 = E.epikv_get_stats(ctx)
+            clocks = Clocks(gpu_id)
+            clocks.start()
+        write_new(K_fill + st * C)
+        E.epikv_set_phase_events(ctx, phase[st])
+        ev[st][0].record(stream)
+        E.epikv_step(ctx, Bn, seq_ids, cu_new, C, budget, trigger, None, view, n_out)
+        ev[st][1].record(stream)
+        n_layer = n_out.cpu().numpy().astype(np.int64)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    E.epikv_set_phase_events(ctx, None)
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    assert (n_layer == np.asarray(budgets)[None, :]).all()
+    stats1 = E.epikv_get_stats(ctx)
+    timed = range(args.warmup, n_steps)
+    ms = sum(ev[i][0].elapsed_time(ev[i][1]) for i in timed)
+    t_score = sum(phase[i][0].elapsed_time(phase[i][1]) for i in timed)
+    t_select = sum(phase[i][1].elapsed_time(phase[i][2]) for i in timed)
+    t_compact = sum(phase[i][2].elapsed_time(phase[i][3]) for i in timed)
+    tokens = stats1["tokens_scored"] - stats0["tokens_scored"]
+    assert tokens == Bn * C * args.steps
+    layer_rows = stats1["layer_rows_moved"] - stats0["layer_rows_moved"]
+    compact_bytes = 2 * layer_rows * 2 * H * d * 2          # read + write of K and V rows of one layer
+    peak, peak_src = measured_hbm_peak()
+    ach = compact_bytes / (t_compact / 1e3) / 1e9
+    line = {
+        "metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"batch{Bn}_32k_lagkv_paged16_layerbudgets_pyramid_mean{K}_chunk{C}",
+                   "sequences": Bn, "layers": L, "kv_heads": H, "head_dim": d, "chunk": C,
+                   "layer_budgets": [budgets[0], budgets[-1]], "budget_mean": K, "score": "lagkv_lag16_w64",
+                   "timing": "sum of per-step device times; each step's new K/V written before it, untimed",
+                   "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
+        "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
+                                "compact": t_compact / args.steps},
+        "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
+                     "frac": ach / peak, "peak_source": peak_src, "traffic": None,
+                     "algorithmic_bytes_per_launch": compact_bytes / args.steps},
+        "gpu_launches": 5 * args.steps,   # Lag-KV partial, finalize, layer keep, layer union, compaction
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -661,6 +797,8 @@ def main():
         run_bandz2k(args)
     elif args.workload == "pertoken":
         run_pertoken(args)
+    elif args.workload == "layers32k":
+        run_layers32k(args)
     else:
         run_ours(args)
 

@@ -131,7 +131,9 @@ size_t carve(const Dims& d, DevState* st, char* base) {
     st->lfirst = (int32_t*)take(S * d.L * 4);
     st->lmask = (unsigned long long*)take(S * T * 8);
     st->lmask_new = (unsigned long long*)take(S * T * 8);
+    st->lkeep = (uint32_t*)take(S * d.L * ((T + 31) / 32) * 4);
     st->mkept = (int32_t*)take(S * T * 4);
+    st->work = (uint32_t*)take(2 * 4);
   }
   return align_up(off, 256);
 }

@@ -59,7 +59,9 @@ struct DevState {
   int32_t* lfirst;         // [S][L] first slot of each layer moved by the last selection
   unsigned long long* lmask;      // [S][T] bit l: layer l holds the token of this slot
   unsigned long long* lmask_new;  // [S][T] the select kernel's new masks (scratch)
+  uint32_t* lkeep;         // [S][L][ceil(T/32)] bit: layer l keeps the union slot (scratch)
   int32_t* mkept;          // [S][T] the select kernel's kept slots of the largest layer (scratch)
+  uint32_t* work;          // [2] the per-layer compaction's next unit and finished CTAs (0 between launches)
 };
 
 struct Dims {

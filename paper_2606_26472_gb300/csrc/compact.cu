@@ -16,6 +16,10 @@
 //
 // Under per-layer budgets (kLayers) each (sequence, layer) has its own kept
 // list, first moved slot and length; the streams and the copy are unchanged.
+// The streams then differ in length (a layer's rows follow its budget), so
+// the CTAs take units from a shared counter instead of a fixed stride, in
+// layer-major order: with budgets that fall with depth, larger streams come
+// first and the greedy assignment ends nearly level.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -107,10 +111,17 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   }
   __syncwarp();
 
+  // the next unit of this CTA: a fixed stride, or the shared counter (kLayers)
+  auto next_unit = [&](int u) -> int {
+    if (!kLayers) return u + G;
+    int v = 0;
+    if (lane == 0) v = (int)atomicAdd(st.work, 1u);
+    return __shfl_sync(0xffffffffu, v, 0);
+  };
   auto load_unit = [&](Cursor& c) {
     while (c.u < units) {
       int e, rem;
-      if (EPIKV_COMPACT_ORDER == 1) {
+      if (kLayers || EPIKV_COMPACT_ORDER == 1) {
         e = c.u % n_ev;
         rem = c.u / n_ev;
       } else {
@@ -130,13 +141,13 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
         c.end = st.n_cache[c.seq];
       }
       if (c.i < c.end) return;
-      c.u += G;
+      c.u = next_unit(c.u);
     }
   };
   auto advance = [&](Cursor& c) {
     c.i += rpb;
     if (c.i >= c.end) {
-      c.u += G;
+      c.u = next_unit(c.u);
       load_unit(c);
     }
   };
@@ -209,7 +220,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   };
 
   Cursor ld;
-  ld.u = blockIdx.x;
+  ld.u = kLayers ? next_unit(0) : (int)blockIdx.x;
   load_unit(ld);
   int pk[kMaxRowsPerLane];
   prefetch(ld, pk);
@@ -250,6 +261,14 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       mbar_wait_bounded(&full[k % kStages], (k / kStages) & 1, kDrainNs);
   }
   tma_wait_all();
+  if (kLayers && lane == 0) {
+    // every CTA has fetched its last unit once all have counted in: the last resets
+    __threadfence();
+    if (atomicAdd(st.work + 1, 1u) == gridDim.x - 1) {
+      st.work[0] = 0u;
+      st.work[1] = 0u;
+    }
+  }
 }
 
 static int g_ctas_per_sm = 0;

@@ -27,11 +27,11 @@
 // cache is always its own budget's selection from any larger layer's cache,
 // so one ranking serves every layer: the context keeps the largest layer's
 // slots (the union of all layers) with a 64-bit mask per slot of the layers
-// holding it.  select_layers_kernel runs one radix select per distinct M_l =
-// K_l - P - R over the union's candidates (largest M first), gives each
-// candidate the mask of the layers whose threshold it passes, and turns the
-// old and new masks into one kept list per layer in that layer's own slot
-// numbering (a block scan per layer), then compacts the union's metadata.
+// holding it.  layer_keep_kernel (a CTA per layer and sequence) finds layer
+// l's threshold of M_l = K_l - P - R over the union's candidates, writes the
+// layer's kept list in its own slot numbering and a keep byte per union slot;
+// layer_union_kernel (a CTA per sequence) turns the keep bytes into the new
+// masks and compacts the union's metadata.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -46,7 +46,8 @@ __device__ __forceinline__ uint32_t order_key(float f) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Exclusive prefix sum over the block; *total receives the sum.
+// Exclusive prefix sum over the block of NT threads; *total receives the sum.
+template <int NT = kSelThreads>
 __device__ __forceinline__ int block_exclusive_scan(int v, int* total, int* sh /*[32]*/) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int x = v;
@@ -58,7 +59,7 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* total, int* sh /
   if (lane == 31) sh[warp] = x;
   __syncthreads();
   if (warp == 0) {
-    int w = lane < (kSelThreads / 32) ? sh[lane] : 0;
+    int w = lane < (NT / 32) ? sh[lane] : 0;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, w, o);
@@ -68,11 +69,12 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* total, int* sh /
   }
   __syncthreads();
   const int before = (warp > 0 ? sh[warp - 1] : 0) + x - v;
-  *total = sh[kSelThreads / 32 - 1];
+  *total = sh[NT / 32 - 1];
   __syncthreads();
   return before;
 }
 
+template <int NT = kSelThreads>
 __device__ __forceinline__ int block_min(int v, int* sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
@@ -80,7 +82,7 @@ __device__ __forceinline__ int block_min(int v, int* sh) {
   if (lane == 0) sh[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    int w = lane < (kSelThreads / 32) ? sh[lane] : INT_MAX;
+    int w = lane < (NT / 32) ? sh[lane] : INT_MAX;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) w = min(w, __shfl_xor_sync(0xffffffffu, w, o));
     if (lane == 0) sh[0] = w;
@@ -99,8 +101,8 @@ struct RadixShared {
 // The M-th largest key_at(i) over i in [c0, c1), 0 < M <= c1 - c0, by a
 // 4-pass 8-bit radix select: *theta is that key and *need_eq the number of
 // keys equal to it that belong to the M largest (the lowest slots first).
-// Every thread of the block calls it.
-template <typename KeyAt>
+// Every thread of the block (NT threads) calls it.
+template <int NT = kSelThreads, typename KeyAt>
 __device__ __forceinline__ void radix_select(const KeyAt& key_at, int c0, int c1, int M, RadixShared& rs,
                                              uint32_t* theta, int* need_eq) {
   const int tid = threadIdx.x;
@@ -111,10 +113,10 @@ __device__ __forceinline__ void radix_select(const KeyAt& key_at, int c0, int c1
     rs.remaining = (uint32_t)M;
   }
   for (int shift = 24; shift >= 0; shift -= 8) {
-    if (tid < 256) rs.hist[tid] = 0u;
+    for (int j = tid; j < 256; j += NT) rs.hist[j] = 0u;
     __syncthreads();
     const uint32_t prefix = rs.prefix, mask = rs.mask;
-    for (int i = c0 + tid; i < c1; i += kSelThreads) {
+    for (int i = c0 + tid; i < c1; i += NT) {
       const uint32_t k = key_at(i);
       if ((k & mask) == prefix) atomicAdd(&rs.hist[(k >> shift) & 255u], 1u);
     }
@@ -293,184 +295,253 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   }
 }
 
-constexpr int kMaxLayers = 64;
+constexpr int kLayerThreads = 256;
 
-__global__ void __launch_bounds__(kSelThreads) select_layers_kernel(DevState st, Dims dm,
-                                                                    const int32_t* __restrict__ seq_ids,
-                                                                    const int32_t* __restrict__ budget,
-                                                                    const int32_t* __restrict__ trigger,
-                                                                    int32_t* __restrict__ kept_out, int kept_stride,
-                                                                    int32_t* __restrict__ n_kept_out) {
-  const int b = blockIdx.x, tid = threadIdx.x, L = dm.L;
+// What both per-layer kernels derive from a sequence's layer budgets.
+// 32-bit words of keep bits per (sequence, layer)
+__host__ __device__ __forceinline__ size_t kKeepWords(int T) { return ((size_t)T + 31) / 32; }
+
+struct LayerEvent {
+  bool event, bad;
+  int n, kmin, kmax, P, R, c0, c1;
+};
+
+__device__ __forceinline__ LayerEvent layer_event(const DevState& st, const Dims& dm, int b, int seq,
+                                                  const int32_t* __restrict__ budget,
+                                                  const int32_t* __restrict__ trigger) {
+  LayerEvent ev;
+  ev.n = st.n_cache[seq];
+  ev.kmin = INT_MAX;
+  ev.kmax = 0;
+  ev.bad = false;
+  for (int l = 0; l < dm.L; ++l) {
+    const int k = budget[(size_t)b * dm.L + l];
+    ev.bad |= k < 1 || k > dm.T;
+    ev.kmin = min(ev.kmin, k);
+    ev.kmax = max(ev.kmax, k);
+  }
+  const int trig = trigger ? trigger[b] : ev.kmax;
+  ev.event = !ev.bad && ev.n > trig && ev.n > ev.kmin;   // some layer is over its budget
+  ev.P = min(st.prefill[seq], ev.n);
+  ev.R = ev.bad ? 0 : min(min(dm.recency_cap, ev.kmin / 4), max(0, ev.kmin - ev.P));
+  ev.c0 = ev.P;
+  ev.c1 = ev.n - ev.R;
+  return ev;
+}
+
+// Ordered passes of the per-layer kernels: warp w of NW owns the slots
+// [w * seg, (w + 1) * seg) and its lanes take 32 consecutive slots at a time
+// (coalesced); lane order inside a group of 32 and the warps' totals, scanned
+// in shared memory, give each slot its rank.
+struct WarpSegment {
+  int lo, hi;
+};
+
+template <int NW>
+__device__ __forceinline__ WarpSegment warp_segment(int n) {
+  const int seg = (n + NW * 32 - 1) / (NW * 32) * 32;
+  const int lo = min(n, (int)(threadIdx.x >> 5) * seg);
+  return WarpSegment{lo, min(n, lo + seg)};
+}
+
+// Exclusive prefix over the warps of per-warp totals v (lane 0's value
+// counts); *total receives the sum.  wt: NW ints of shared memory.
+template <int NW>
+__device__ __forceinline__ int warp_base(int v, int* total, int* wt) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) wt[warp] = v;
+  __syncthreads();
+  int before = 0, all = 0;
+  for (int w = 0; w < NW; ++w) {
+    before += w < warp ? wt[w] : 0;
+    all += wt[w];
+  }
+  __syncthreads();
+  *total = all;
+  return before;
+}
+
+// Per-layer selection, one CTA per (layer, batch entry): layer l's M_l =
+// K_l - P - R best candidates of the union (a radix select on the union's
+// candidates), its kept list in its own slot numbering, its new length and
+// first moved slot, and one bit per union slot saying whether the layer
+// keeps it (a 32-bit word per 32 slots, read by layer_union_kernel).
+__global__ void __launch_bounds__(kLayerThreads) layer_keep_kernel(DevState st, Dims dm,
+                                                                   const int32_t* __restrict__ seq_ids,
+                                                                   const int32_t* __restrict__ budget,
+                                                                   const int32_t* __restrict__ trigger,
+                                                                   int32_t* __restrict__ kept_out, int kept_stride,
+                                                                   int32_t* __restrict__ n_kept_out) {
+  constexpr int NT = kLayerThreads, NW = NT / 32;
+  const int l = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, L = dm.L;
+  const int lane = tid & 31;
+  const unsigned lt = (1u << lane) - 1u;
   const int seq = seq_ids[b];
   if (seq < 0 || seq >= dm.S) {
-    if (tid == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    if (tid == 0 && l == 0) set_error(st.err, EPIKV_DEV_BATCH);
     return;
   }
-  __shared__ int sK[kMaxLayers];
-  __shared__ int s_bad, s_changed, s_ng;
-  __shared__ int s_gM[kMaxLayers];
-  __shared__ unsigned long long s_gbits[kMaxLayers];
   __shared__ RadixShared rs;
   __shared__ int sh_scan[32];
-  int32_t* nl = st.n_layer + (size_t)seq * L;
-  int32_t* lf = st.lfirst + (size_t)seq * L;
-  const int n = st.n_cache[seq];
-  if (tid == 0) {
-    s_bad = 0;
-    s_changed = 0;
-  }
-  __syncthreads();
-  if (tid < L) {
-    const int k = budget[(size_t)b * L + tid];
-    sK[tid] = k;
-    if (k < 1 || k > dm.T) atomicOr(&s_bad, 1);
-  }
-  __syncthreads();
-  // no event: every layer keeps what it holds
-  auto keep_all = [&]() {
-    for (int l = tid; l < L; l += kSelThreads) {
-      lf[l] = nl[l];
-      if (n_kept_out) n_kept_out[(size_t)b * L + l] = nl[l];
+  __shared__ int wt[NW];
+  int32_t* nl = st.n_layer + (size_t)seq * L + l;
+  int32_t* lf = st.lfirst + (size_t)seq * L + l;
+  const LayerEvent ev = layer_event(st, dm, b, seq, budget, trigger);
+  if (ev.bad && tid == 0 && l == 0) set_error(st.err, EPIKV_DEV_BUDGET);
+  const bool fits = max(ev.kmax, ev.P) <= kept_stride;
+  if (ev.event && !fits && tid == 0 && l == 0) set_error(st.err, EPIKV_DEV_KEPT);
+  if (!ev.event || !fits) {  // every layer keeps what it holds
+    if (tid == 0) {
+      *lf = *nl;
+      if (n_kept_out) n_kept_out[(size_t)b * L + l] = *nl;
     }
-    if (tid == 0) st.first_changed[seq] = n;
-  };
-  if (s_bad) {
-    if (tid == 0) set_error(st.err, EPIKV_DEV_BUDGET);
-    keep_all();
     return;
   }
-  int kmin = INT_MAX, kmax = 0;
-  for (int l = 0; l < L; ++l) {
-    kmin = min(kmin, sK[l]);
-    kmax = max(kmax, sK[l]);
-  }
-  const int trig = trigger ? trigger[b] : kmax;
-  if (n <= trig || n <= kmin) {  // no layer is over its budget, or no event yet
-    keep_all();
-    return;
-  }
-  const int P = min(st.prefill[seq], n);
-  const int R = min(min(dm.recency_cap, kmin / 4), max(0, kmin - P));
-  const int c0 = P, c1 = n - R;  // the union's candidates [c0, c1)
-  if (max(kmax, P) > kept_stride) {
-    if (tid == 0) set_error(st.err, EPIKV_DEV_KEPT);
-    keep_all();
-    return;
-  }
+  const int n = ev.n, c0 = ev.c0, c1 = ev.c1;
+  const int M = max(0, budget[(size_t)b * L + l] - ev.P - ev.R);
   const float* __restrict__ sc = st.score[kind_index(st.policy[seq])] + (size_t)seq * dm.T;
-  unsigned long long* __restrict__ mk = st.lmask + (size_t)seq * dm.T;
-  unsigned long long* __restrict__ mn = st.lmask_new + (size_t)seq * dm.T;
+  const unsigned long long* __restrict__ mk = st.lmask + (size_t)seq * dm.T;
+  uint32_t* __restrict__ keep = st.lkeep + ((size_t)seq * L + l) * kKeepWords(dm.T);
   auto key_at = [&](int i) -> uint32_t { return order_key(sc[i]); };
 
-  // ---- layers grouped by equal M_l, largest M first; s_gbits[g] holds the
-  // layers of groups 0..g (those that keep a candidate group g keeps)
+  // threshold of this layer's M best candidates
+  uint32_t theta = 0xFFFFFFFFu;
+  int need_eq = 0;
+  const bool all = M >= c1 - c0;  // every candidate passes
+  const bool sel = M > 0 && !all;
+  if (sel) radix_select<NT>(key_at, c0, c1, M, rs, &theta, &need_eq);
+
+  const WarpSegment sg = warp_segment<NW>(n);
+  // pass 1: per-warp counts of candidates equal to theta and of held slots
+  int ceq = 0, cold = 0;
+  for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
+    const int i = i0 + lane;
+    const bool in = i < sg.hi;
+    const bool eq = sel && in && i >= c0 && i < c1 && key_at(i) == theta;
+    const bool held = in && ((mk[i] >> l) & 1ull);
+    ceq += __popc(__ballot_sync(0xffffffffu, eq));
+    cold += __popc(__ballot_sync(0xffffffffu, held));
+  }
+  int n_eq, n_old;
+  int q = warp_base<NW>(ceq, &n_eq, wt);
+  const int old_base = warp_base<NW>(cold, &n_old, wt);
+  // pass 2: the layer's decision per slot (a keep byte), per-warp kept counts
+  int cnew = 0;
+  for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
+    const int i = i0 + lane;
+    const bool in = i < sg.hi;
+    const bool cand = in && i >= c0 && i < c1;
+    const bool held = in && ((mk[i] >> l) & 1ull);
+    uint32_t key = 0u;
+    if (cand && sel) key = key_at(i);
+    const bool eq = cand && sel && key == theta;
+    const unsigned eb = __ballot_sync(0xffffffffu, eq);
+    const int rank = q + __popc(eb & lt);  // among the candidates equal to theta, in slot order
+    q += __popc(eb);
+    bool k = held;
+    if (cand) {
+      const bool pass = all || (sel && (key > theta || (eq && rank < need_eq)));
+      if (pass && !held) set_error(st.err, EPIKV_DEV_KEPT);  // the layers' caches are not nested
+      k = pass && held;
+    }
+    const unsigned kb = __ballot_sync(0xffffffffu, k);
+    if (lane == 0) keep[i0 >> 5] = kb;  // segments start at multiples of 32
+    cnew += __popc(kb);
+  }
+  int n_new;
+  int j = warp_base<NW>(cnew, &n_new, wt);
+  // pass 3: the kept list, old slot numbers in new slot order
+  int32_t* out = kept_out + ((size_t)b * L + l) * kept_stride;
+  int o = old_base, fe = INT_MAX;
+  for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
+    const int i = i0 + lane;
+    const bool in = i < sg.hi;
+    const bool held = in && ((mk[i] >> l) & 1ull);
+    const unsigned kb = keep[i0 >> 5];
+    const bool k = (kb >> lane) & 1u;
+    const unsigned hb = __ballot_sync(0xffffffffu, held);
+    if (k) {
+      const int my_o = o + __popc(hb & lt), my_j = j + __popc(kb & lt);
+      if (my_j < kept_stride) out[my_j] = my_o;
+      if (my_o != my_j) fe = min(fe, my_j);
+    }
+    o += __popc(hb);
+    j += __popc(kb);
+  }
+  fe = block_min<NT>(fe, sh_scan);
   if (tid == 0) {
-    int ord[kMaxLayers];
-    for (int l = 0; l < L; ++l) {
-      const int m = max(0, sK[l] - P - R);
-      int j = l;
-      while (j > 0 && max(0, sK[ord[j - 1]] - P - R) < m) {
-        ord[j] = ord[j - 1];
-        --j;
-      }
-      ord[j] = l;
-    }
-    int ng = 0;
-    unsigned long long bits = 0ull;
-    for (int j = 0; j < L; ++j) {
-      const int m = max(0, sK[ord[j]] - P - R);
-      if (j > 0 && m != s_gM[ng - 1]) ++ng;
-      if (j == 0) ng = 1;
-      s_gM[ng - 1] = m;
-      bits |= 1ull << ord[j];
-      s_gbits[ng - 1] = bits;
-    }
-    s_ng = ng;
+    if (n_old != *nl) set_error(st.err, EPIKV_DEV_KEPT);  // the masks and the length disagree
+    const int f = min(fe, n_new);
+    *lf = f;
+    *nl = n_new;
+    if (n_kept_out) n_kept_out[(size_t)b * L + l] = n_new;
+    atomicAdd(&st.stats[3], (unsigned long long)(n_new - f));
   }
-  // protected slots keep their layers; candidates start with none
-  for (int i = tid; i < n; i += kSelThreads) mn[i] = (i < c0 || i >= c1) ? mk[i] : 0ull;
-  __syncthreads();
+}
 
-  const int ncand = c1 - c0;
-  const int per = (n + kSelThreads - 1) / kSelThreads;
-  const int a = min(n, tid * per), e = min(n, a + per);
-  for (int g = 0; g < s_ng; ++g) {
-    const int M = s_gM[g];
-    const unsigned long long bits = s_gbits[g];
-    if (M <= 0) break;  // this group and the smaller ones keep no candidate
-    if (M >= ncand) {   // every candidate passes
-      for (int i = c0 + tid; i < c1; i += kSelThreads) mn[i] = bits;
-      __syncthreads();
-      continue;
-    }
-    uint32_t theta;
-    int need_eq;
-    radix_select(key_at, c0, c1, M, rs, &theta, &need_eq);
-    int eq_local = 0;
-    for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (key_at(i) == theta);
-    int tot;
-    int eqs = block_exclusive_scan(eq_local, &tot, sh_scan);
-    for (int i = max(a, c0); i < min(e, c1); ++i) {
-      const uint32_t k = key_at(i);
-      if (k > theta || (k == theta && eqs++ < need_eq)) mn[i] = bits;
-    }
-    __syncthreads();
+// The union of the layers after a per-layer selection, one CTA per batch
+// entry: each slot's new layer mask (from the keep bytes), the kept slots of
+// the union (the largest layer's), and the in-place compaction of the slot
+// metadata (scores, positions, masks).
+__global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, Dims dm,
+                                                                  const int32_t* __restrict__ seq_ids,
+                                                                  const int32_t* __restrict__ budget,
+                                                                  const int32_t* __restrict__ trigger,
+                                                                  int kept_stride) {
+  constexpr int NW = kSelThreads / 32;
+  const int b = blockIdx.x, tid = threadIdx.x, L = dm.L;
+  const int lane = tid & 31;
+  const unsigned lt = (1u << lane) - 1u;
+  const int seq = seq_ids[b];
+  if (seq < 0 || seq >= dm.S) return;   // reported by layer_keep_kernel
+  __shared__ int sh_scan[32];
+  __shared__ int wt[NW];
+  __shared__ int s_changed;
+  const LayerEvent ev = layer_event(st, dm, b, seq, budget, trigger);
+  const int n = ev.n;
+  if (!ev.event || max(ev.kmax, ev.P) > kept_stride) {
+    if (tid == 0) st.first_changed[seq] = n;
+    return;
   }
-  // a layer keeps only tokens it holds (true by the nesting; checked)
-  for (int i = c0 + tid; i < c1; i += kSelThreads) {
-    const unsigned long long nm = mn[i], om = mk[i];
-    if (nm & ~om) set_error(st.err, EPIKV_DEV_KEPT);
-    mn[i] = nm & om;
+  unsigned long long* __restrict__ mk = st.lmask + (size_t)seq * dm.T;
+  unsigned long long* __restrict__ mn = st.lmask_new + (size_t)seq * dm.T;
+  const uint32_t* __restrict__ keep = st.lkeep + (size_t)seq * L * kKeepWords(dm.T);
+  const size_t kw = kKeepWords(dm.T);
+  if (tid == 0) {
+    int ch = 0;
+    for (int l = 0; l < L; ++l) ch |= st.lfirst[(size_t)seq * L + l] < st.n_layer[(size_t)seq * L + l];
+    s_changed = ch;
+  }
+  // new masks: a warp takes 32 consecutive slots and one keep word per layer
+  for (int i0 = (tid >> 5) * 32; i0 < n; i0 += kSelThreads) {
+    const int i = i0 + lane;
+    unsigned long long m = 0ull;
+#pragma unroll 8
+    for (int l = 0; l < L; ++l) m |= (unsigned long long)((keep[l * kw + (i0 >> 5)] >> lane) & 1u) << l;
+    if (i < n) mn[i] = m;
   }
   __syncthreads();
-
-  // ---- one kept list per layer, in that layer's slot numbering
-  unsigned long long moved = 0ull;
-  for (int l = 0; l < L; ++l) {
-    int co = 0, cn = 0;
-    for (int i = a; i < e; ++i) {
-      co += (int)((mk[i] >> l) & 1ull);
-      cn += (int)((mn[i] >> l) & 1ull);
-    }
-    int n_old, n_new;
-    int o = block_exclusive_scan(co, &n_old, sh_scan);
-    int j = block_exclusive_scan(cn, &n_new, sh_scan);
-    int32_t* out = kept_out + ((size_t)b * L + l) * kept_stride;
-    int fe = INT_MAX;
-    for (int i = a; i < e; ++i) {
-      if ((mn[i] >> l) & 1ull) {
-        if (j < kept_stride) out[j] = o;
-        if (o != j) fe = min(fe, j);
-        ++j;
-      }
-      if ((mk[i] >> l) & 1ull) ++o;
-    }
-    fe = block_min(fe, sh_scan);
-    if (tid == 0) {
-      if (n_old != nl[l]) set_error(st.err, EPIKV_DEV_KEPT);  // masks and length disagree
-      const int f = min(fe, n_new);
-      lf[l] = f;
-      nl[l] = n_new;
-      if (n_kept_out) n_kept_out[(size_t)b * L + l] = n_new;
-      moved += (unsigned long long)(n_new - f);
-      if (f < n_new) s_changed = 1;
-    }
-  }
-
-  // ---- the union's kept slots (any layer holds them), then its metadata
-  int32_t* mkept = st.mkept + (size_t)seq * dm.T;
+  const WarpSegment sg = warp_segment<NW>(n);
   int cu = 0;
-  for (int i = a; i < e; ++i) cu += mn[i] != 0ull;
+  for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
+    const int i = i0 + lane;
+    cu += __popc(__ballot_sync(0xffffffffu, i < sg.hi && mn[i] != 0ull));
+  }
   int n_union;
-  int o = block_exclusive_scan(cu, &n_union, sh_scan);
+  int o = warp_base<NW>(cu, &n_union, wt);
+  int32_t* mkept = st.mkept + (size_t)seq * dm.T;
   int fe = INT_MAX;
-  for (int i = a; i < e; ++i)
-    if (mn[i] != 0ull) {
-      mkept[o] = i;
-      if (o != i) fe = min(fe, o);
-      ++o;
+  for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
+    const int i = i0 + lane;
+    const bool k = i < sg.hi && mn[i] != 0ull;
+    const unsigned kb = __ballot_sync(0xffffffffu, k);
+    if (k) {
+      const int my_o = o + __popc(kb & lt);
+      mkept[my_o] = i;
+      if (my_o != i) fe = min(fe, my_o);
     }
+    o += __popc(kb);
+  }
   fe = min(block_min(fe, sh_scan), n_union);
   __syncthreads();  // the union's kept list is visible to the whole block
   int32_t* ps = st.pos + (size_t)seq * dm.T;
@@ -493,15 +564,13 @@ __global__ void __launch_bounds__(kSelThreads) select_layers_kernel(DevState st,
     }
     __syncthreads();
   }
-  // every new mask lands in its slot (the ones before fe did not move)
+  // every new mask lands in its slot (the slots before fe did not move)
   for (int j = tid; j < n_union; j += kSelThreads) mk[j] = mn[mkept[j]];
-  __syncthreads();
   if (tid == 0) {
     st.n_cache[seq] = n_union;
     st.first_changed[seq] = s_changed ? 0 : n_union;
     atomicAdd(&st.stats[1], 1ull);
     atomicAdd(&st.stats[2], (unsigned long long)(n_union - fe));
-    atomicAdd(&st.stats[3], moved);
   }
 }
 
@@ -509,10 +578,14 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
                           const int32_t* budget, const int32_t* trigger, int32_t* kept, int kept_stride,
                           int32_t* n_kept, cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
-  if (dm.layer_budgets)
-    select_layers_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
-                                                            n_kept);
-  else if (dm.select_chunk > 1)
+  if (dm.layer_budgets) {
+    layer_keep_kernel<<<dim3(dm.L, n_seq), kLayerThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept,
+                                                                       kept_stride, n_kept);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    ++*launches;
+    layer_union_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept_stride);
+  } else if (dm.select_chunk > 1)
     select_kernel<true><<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
                                                            n_kept);
   else

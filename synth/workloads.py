@@ -80,3 +80,15 @@ def small_model(seed: int) -> TraceModel:
     """A reduced model for parity tests that the oracle finishes in seconds."""
     return TraceModel(seed, num_layers=4, hidden=256, num_kv_heads=2, head_dim=32,
                       band_a=(1,), band_b=(2, 3))
+
+
+def pyramid_budgets(k_mean: int, n_layers: int, spread: float = 0.5, multiple: int = 16) -> tuple:
+    """A per-layer budget vector for the per-layer budget workloads: larger
+    budgets for lower layers, falling linearly from (1 + spread) * k_mean at
+    layer 0 to (1 - spread) * k_mean at the last layer, each rounded to a
+    multiple of ``multiple`` (so the mean stays k_mean)."""
+    out = []
+    for l in range(n_layers):
+        f = 1.0 + spread * (1.0 - 2.0 * l / (n_layers - 1)) if n_layers > 1 else 1.0
+        out.append(int(round(k_mean * f / multiple)) * multiple)
+    return tuple(out)

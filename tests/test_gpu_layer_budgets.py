@@ -11,6 +11,7 @@ import pytest
 from oracle import epikv_oracle as O
 from paper_2606_26472_gb300 import epikv as E
 from synth import gen, workloads as W
+from synth.device import as_u16
 
 from .harness import OracleTrace, Session, assert_scores_close
 
@@ -187,4 +188,57 @@ def test_a_bad_layer_budget_is_reported_and_nothing_moves(gpu_lib):
     assert sess.error() == (E.EPIKV_EDEVICE, E.EPIKV_DEV_BUDGET)
     for l in range(model.num_layers):
         np.testing.assert_array_equal(sess.read_layer(0, l), before[l])
+    sess.close()
+
+
+def test_config2_shape_with_pyramid_layer_budgets(gpu_lib):
+    """The 8 x 8,192 band-z workload (32 layers, 64 new tokens per call, the
+    trigger K_max + 63) with pyramid per-layer budgets 6,144 .. 2,048 (mean
+    4,096): every layer's positions of two sequences equal the oracle's
+    replay after the first event, mid-way and at the end; every layer ends at
+    its budget; sampled slots of every layer hold the generator's rows."""
+    wl = W.config(2)
+    m = wl.model
+    L = m.num_layers
+    budgets = W.pyramid_budgets(wl.budgets[0], L)
+    K_max = max(budgets)
+    sess = Session(m, n_seq=wl.n_seq, kinds=wl.kinds, layout=wl.layout, max_tokens=K_max + wl.chunk,
+                   max_new=wl.chunk, prefill=[0] * wl.n_seq, policies=wl.policies, layer_budgets=1)
+    trig = K_max + wl.trigger_slack[0]
+    checked = (0, 5)
+    replay = {b: LayerReplay(L, budgets, 0, trig) for b in checked}
+    n_steps = wl.max_len // wl.chunk
+    first = trig // wl.chunk                  # the first step that evicts
+    rng = np.random.default_rng(7)
+    events = 0
+    for st in range(n_steps):
+        entries = [(b, wl.chunk) for b in range(wl.n_seq)]
+        before = {b: sess.n_cache[b] for b in checked}
+        sess.score_update(entries)
+        for b in checked:
+            pos, sc = sess.read(b, sess.policies[b])
+            new = slice(before[b], before[b] + wl.chunk)
+            replay[b].append(pos[new], sc[new])
+        kept = sess.select(list(range(wl.n_seq)), [list(budgets)] * wl.n_seq, [trig] * wl.n_seq)
+        sess.compact(list(range(wl.n_seq)))
+        for b in checked:
+            events += replay[b].event()
+        if st >= first:
+            assert len(kept) == wl.n_seq, f"step {st}: every sequence evicts"
+        if st in (first, 110, n_steps - 1):
+            for b in checked:
+                for l in range(L):
+                    assert list(sess.read_layer(b, l)) == replay[b].caches[l], f"step {st} seq {b} layer {l}"
+    assert events == 2 * (n_steps - first)
+    assert all(sess.n_layer[b] == list(budgets) for b in range(wl.n_seq))
+    for b in checked:
+        slots = np.sort(rng.choice(min(budgets), size=24, replace=False))
+        k = as_u16(sess.cache.rows(0, b, slots, sess.bt_host))
+        v = as_u16(sess.cache.rows(1, b, slots, sess.bt_host))
+        sp = gen.spike_flags(m, b, wl.max_len)
+        for l in range(L):
+            pos = np.asarray(replay[b].caches[l])[slots]
+            np.testing.assert_array_equal(k[:, l], gen.kv_rows(m, sess.dt.tabs, b, 0, pos, sp)[:, l])
+            np.testing.assert_array_equal(v[:, l], gen.kv_rows(m, sess.dt.tabs, b, 1, pos, sp)[:, l])
+    assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()
