@@ -193,14 +193,91 @@ __device__ __forceinline__ uint4 q_max(const uint4& a, const uint4& b) {
   return make_uint4(bf16x2_max(a.x, b.x), bf16x2_max(a.y, b.y), bf16x2_max(a.z, b.z), bf16x2_max(a.w, b.w));
 }
 
-// Minimum and reciprocal range denominator of the previous chunk, per channel.
-__device__ __forceinline__ void prev_range(const uint4& pmn, const uint4& pmx, float eps, float (&mn)[8],
-                                           float (&inv)[8]) {
-  float mx[8];
+// ---- packed fp32 pairs: Blackwell's f32x2 arithmetic, two channels per instruction
+typedef unsigned long long f32x2;
+
+__device__ __forceinline__ f32x2 f2_pack(float lo, float hi) {
+  return ((f32x2)__float_as_uint(hi) << 32) | (f32x2)__float_as_uint(lo);
+}
+__device__ __forceinline__ float f2_lo(f32x2 v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float f2_hi(f32x2 v) { return __uint_as_float((uint32_t)(v >> 32)); }
+__device__ __forceinline__ f32x2 f2_fma(f32x2 a, f32x2 b, f32x2 c) {
+  f32x2 d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ f32x2 f2_add(f32x2 a, f32x2 b) {
+  f32x2 d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ f32x2 f2_mul(f32x2 a, f32x2 b) {
+  f32x2 d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// the two bf16 channels of a 32-bit word as an fp32 pair (exact)
+__device__ __forceinline__ f32x2 bf16x2_to_f2(uint32_t w) { return f2_pack(bf16_lo(w), bf16_hi(w)); }
+
+// The previous chunk's range as a per-channel affine map y = x * a + c with
+// a = 1 / (max - min + eps) and c = -min * a - 1/2, so that y = x~ - 1/2 for
+// the range-normalised x~ (one fused multiply-add per channel).
+__device__ __forceinline__ void prev_affine(const uint4& pmn, const uint4& pmx, float eps, f32x2 (&a)[4],
+                                            f32x2 (&c)[4]) {
+  float mn[8], mx[8], inv[8], bias[8];
   unpack8(pmn, mn);
   unpack8(pmx, mx);
 #pragma unroll
-  for (int e = 0; e < 8; ++e) inv[e] = 1.f / (mx[e] - mn[e] + eps);
+  for (int e = 0; e < 8; ++e) {
+    inv[e] = 1.f / (mx[e] - mn[e] + eps);
+    bias[e] = fmaf(-mn[e], inv[e], -0.5f);
+  }
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    a[p] = f2_pack(inv[2 * p], inv[2 * p + 1]);
+    c[p] = f2_pack(bias[2 * p], bias[2 * p + 1]);
+  }
+}
+
+// Sums of y and y^2 over one thread's 8 channels of a token row.
+__device__ __forceinline__ void lag_moments(const uint4& x, const f32x2 (&a)[4], const f32x2 (&c)[4], float& s1,
+                                            float& s2) {
+  const f32x2 y0 = f2_fma(bf16x2_to_f2(x.x), a[0], c[0]);
+  const f32x2 y1 = f2_fma(bf16x2_to_f2(x.y), a[1], c[1]);
+  const f32x2 y2 = f2_fma(bf16x2_to_f2(x.z), a[2], c[2]);
+  const f32x2 y3 = f2_fma(bf16x2_to_f2(x.w), a[3], c[3]);
+  const f32x2 t = f2_add(f2_add(y0, y1), f2_add(y2, y3));
+  f32x2 u = f2_mul(y0, y0);
+  u = f2_fma(y1, y1, u);
+  u = f2_fma(y2, y2, u);
+  u = f2_fma(y3, y3, u);
+  s1 = f2_lo(t) + f2_hi(t);
+  s2 = f2_lo(u) + f2_hi(u);
+}
+
+// Transposed sum over the O*2 lanes of a group: every level halves the values
+// a lane keeps and sends the other half to its partner, so NV values cost
+// NV - 1 shuffles in all instead of one butterfly of log2(lanes) shuffles per
+// value.  With lanes <= NV, value k + (NV / lanes) * (lane % lanes) ends in
+// v[k]; with more lanes than values, value (lane % lanes) / (lanes / NV) ends
+// in v[0].
+template <int O, int C, int NV>
+__device__ __forceinline__ void transpose_sum(float (&v)[NV], int lane) {
+  if constexpr (O >= 1) {
+    if constexpr (C > 1) {
+      const bool up = lane & O;
+#pragma unroll
+      for (int k = 0; k < C / 2; ++k) {
+        const float send = up ? v[k] : v[k + C / 2];
+        const float keep = up ? v[k + C / 2] : v[k];
+        v[k] = keep + __shfl_xor_sync(0xffffffffu, send, O);
+      }
+      transpose_sum<O / 2, C / 2, NV>(v, lane);
+    } else {
+      v[0] += __shfl_xor_sync(0xffffffffu, v[0], O);
+      transpose_sum<O / 2, 1, NV>(v, lane);
+    }
+  }
 }
 
 // grid: (2L (layer, K|V), batch entries); block: max(32, H*d/8) threads;
@@ -211,7 +288,9 @@ __device__ __forceinline__ void prev_range(const uint4& pmn, const uint4& pmx, f
 // reductions are independent of one another.  Chunk ranges (min, max) are
 // bf16 values and are kept packed (exact).  The variance of a token's head
 // is taken from the moments of y = x~ - 1/2 (x~ in [0, 1] inside the range),
-// one two-value group reduction per token.
+// computed two channels per instruction (f32x2); the segment's 2 x 8 moments
+// are summed over the head's lanes by one transposed reduction into shared
+// memory, where a thread per token forms each head's variance.
 template <int LH>
 __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
                                                              const int32_t* __restrict__ seq_ids,
@@ -248,13 +327,14 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
     cmn = *reinterpret_cast<const uint4*>(rng + 2 * hd + ch);
     cmx = *reinterpret_cast<const uint4*>(rng + 3 * hd + ch);
   }
-  float mn[8], inv[8];
-  prev_range(pmn, pmx, dm.lag_eps, mn, inv);
+  f32x2 na[4], nc[4];
+  prev_affine(pmn, pmx, dm.lag_eps, na, nc);
 
   const float inv_d = 1.f / (float)dm.d;
   const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
   __shared__ int64_t soff[kLagOffs];
-  __shared__ float hv[2][kLagSeg][32];  // [segment parity][token][head]; the host admits H <= 32
+  constexpr int NV = 2 * kLagSeg;      // moments of a segment: (sum y, sum y^2) per token
+  __shared__ float red[2][32][NV];      // [segment parity][head][moment]; the host admits H <= 32
   __shared__ float hr[2][kLagSeg][32];  // raw variances, same layout
   float* part = need_norm ? st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
   float* rpart = need_raw ? st.raw_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
@@ -299,25 +379,23 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
             const float var_raw = group_sum(s2, LH) * inv_d;
             if (q == 0 && active) hr[parity][j][h] = var_raw;
           }
-          float var = 0.f;
-          if (has_prev && need_norm) {  // uniform across the block
-            float xf[8], s1 = 0.f, s2 = 0.f;
-            unpack8(x[j], xf);
+        }
+      }
+      if (has_prev && need_norm) {  // uniform across the block
+        float v[NV];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float y = fmaf(xf[e] - mn[e], inv[e], -0.5f);
-              s1 += y;
-              s2 = fmaf(y, y, s2);
-            }
+        for (int j = 0; j < kLagSeg; ++j) {
+          v[2 * j] = v[2 * j + 1] = 0.f;
+          if (j < seg) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
+        }
+        transpose_sum<LH / 2, NV, NV>(v, tid & 31);
+        if (active) {
+          if constexpr (LH <= NV) {
 #pragma unroll
-            for (int o = LH >> 1; o > 0; o >>= 1) {
-              s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-              s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-            }
-            const float mean = s1 * inv_d;
-            var = fmaxf(fmaf(-mean, mean, s2 * inv_d), 0.f);
+            for (int k = 0; k < NV / LH; ++k) red[parity][h][k + (NV / LH) * q] = v[k];
+          } else {
+            if (q % (LH / NV) == 0) red[parity][h][q / (LH / NV)] = v[0];
           }
-          if (q == 0 && active) hv[parity][j][h] = var;
         }
       }
       // advance the running range of the current chunk
@@ -335,7 +413,11 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
       if (tid < seg) {
         if (need_norm) {
           float sum = 0.f;
-          for (int hh = 0; hh < dm.H; ++hh) sum += hv[parity][tid][hh];
+          if (has_prev)
+            for (int hh = 0; hh < dm.H; ++hh) {
+              const float mean = red[parity][hh][2 * tid] * inv_d;
+              sum += fmaxf(fmaf(-mean, mean, red[parity][hh][2 * tid + 1] * inv_d), 0.f);
+            }
           part[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
         }
         if (need_raw) {
@@ -349,7 +431,7 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
       if (r == dm.lag) {  // chunk complete: it becomes the previous chunk
         pmn = cmn;
         pmx = cmx;
-        prev_range(pmn, pmx, dm.lag_eps, mn, inv);
+        prev_affine(pmn, pmx, dm.lag_eps, na, nc);
         r = 0;
       }
       i += seg;
