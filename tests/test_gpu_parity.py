@@ -45,6 +45,9 @@ CASES = [
      (1, 9, 64), 5, 1),
     ("contig_all_kinds_a", E.EPIKV_LAYOUT_CONTIGUOUS, 63, (0, 2, 0), (90, 70, 110), (5, 16, 23), 16, 1),
     ("paged_all_kinds_b", E.EPIKV_LAYOUT_PAGED, 63, (0, 0, 9), (60, 100, 75), (32, 3, 12), 7, 1),
+    # long prefixes: P = 100 < K, P = 1, and P = 100 > K (the whole prefill kept, no recency window)
+    ("contig_bandz_prefill100", E.EPIKV_LAYOUT_CONTIGUOUS, E.EPIKV_SCORE_BANDZ, (100, 1, 100), (150, 64, 64),
+     (7, 1, 33), 16, 1),
     # chunk-level selection
     ("contig_bandz_chunk4", E.EPIKV_LAYOUT_CONTIGUOUS, E.EPIKV_SCORE_BANDZ, (0, 5, 0), (100, 60, 130), (7, 1, 33),
      16, 4),
