@@ -134,9 +134,14 @@ typedef struct {
 
 /* The K/V cache (Sec. 3.1: 2*L*H*d scalars per token).  Element offsets:
  *   contiguous: layer*stride_layer + seq*stride_seq + slot*stride_token
- *   paged:      layer*stride_layer + block_table[seq*max_blocks_per_seq +
- *               slot/block_size]*stride_block + (slot%block_size)*stride_token
- * The same offsets address k and v. */
+ *   paged:      layer*stride_layer + block_table[layer*stride_table_layer +
+ *               seq*max_blocks_per_seq + slot/block_size]*stride_block +
+ *               (slot%block_size)*stride_token
+ * The same offsets address k and v.  stride_table_layer = 0 shares one block
+ * table among the layers; with per-layer budgets, stride_layer = 0 and one
+ * table per layer describe a single pool of blocks in which every (layer,
+ * sequence) owns its own blocks, so each layer's memory follows its own
+ * budget.  The caller keeps distinct (layer, sequence) block lists disjoint. */
 typedef struct {
   void* k;
   void* v;
@@ -149,6 +154,8 @@ typedef struct {
   int32_t max_blocks_per_seq;   /* paged only */
   int32_t block_size;           /* paged only: tokens per block */
   int32_t num_blocks;           /* paged only: pool size, for bounds checks */
+  int64_t stride_table_layer;   /* paged only: elements between consecutive layers' block
+                                 * tables (0: one table for every layer) */
 } epikv_kv_view;
 
 typedef struct {

@@ -157,8 +157,9 @@ bool valid_kv(const epikv_ctx* ctx, const epikv_kv_view* kv, KvDev* out) {
   }
   if (kv->layout != EPIKV_LAYOUT_PAGED) return false;
   if (!kv->block_table || kv->block_size < 1 || kv->max_blocks_per_seq < 1 || kv->num_blocks < 1) return false;
-  if (kv->stride_block < 0 || kv->stride_block % 8) return false;
+  if (kv->stride_block < 0 || kv->stride_block % 8 || kv->stride_table_layer < 0) return false;
   out->stride_block = kv->stride_block;
+  out->table_stride_layer = kv->stride_table_layer;
   out->block_table = kv->block_table;
   out->max_blocks = kv->max_blocks_per_seq;
   out->block_size = kv->block_size;

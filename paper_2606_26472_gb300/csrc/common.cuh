@@ -76,6 +76,7 @@ struct KvDev {
   int64_t stride_layer, stride_seq, stride_block, stride_token;  // elements
   const int32_t* block_table;
   int max_blocks, block_size, num_blocks;
+  int64_t table_stride_layer;  // elements between layers' block tables (0: shared)
 };
 
 __device__ __forceinline__ void set_error(int32_t* err, int code) {
@@ -91,7 +92,7 @@ __device__ __forceinline__ int64_t kv_row_offset(const KvDev& v, int layer, int 
   }
   int bi = slot / v.block_size;
   if (bi >= v.max_blocks) return -1;
-  int blk = __ldg(v.block_table + (int64_t)seq * v.max_blocks + bi);
+  int blk = __ldg(v.block_table + (int64_t)layer * v.table_stride_layer + (int64_t)seq * v.max_blocks + bi);
   if (blk < 0 || blk >= v.num_blocks) return -1;
   return (int64_t)layer * v.stride_layer + (int64_t)blk * v.stride_block +
          (int64_t)(slot - bi * v.block_size) * v.stride_token;

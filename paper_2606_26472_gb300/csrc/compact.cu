@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       pk[j] = r < nrows ? __ldg(kl + r) : 0;
     }
   };
-  int staged_seq = -1;
+  int staged_seq = -1, staged_layer = -1;
   // element offset of a slot of the current sequence, -1 outside the view
   auto slot_offset = [&](int layer, int seq, int slot) -> int64_t {
     if (!bt_in_smem) return kv_row_offset(kv, layer, seq, slot, dm.T);
@@ -177,11 +177,14 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
 
   // issue the loads of the batch at cursor c (kept slots pk) into stage s
   auto issue = [&](const Cursor& c, const int (&pk)[kMaxRowsPerLane], int s) {
-    if (bt_in_smem && c.seq != staged_seq) {
+    // the stream's block table (per layer when the layers have their own tables)
+    if (bt_in_smem && (c.seq != staged_seq || (kv.table_stride_layer && c.layer != staged_layer))) {
       __syncwarp();
-      for (int j = lane; j < kv.max_blocks; j += 32) bt_s[j] = __ldg(kv.block_table + (int64_t)c.seq * kv.max_blocks + j);
+      const int32_t* tab = kv.block_table + (int64_t)c.layer * kv.table_stride_layer + (int64_t)c.seq * kv.max_blocks;
+      for (int j = lane; j < kv.max_blocks; j += 32) bt_s[j] = __ldg(tab + j);
       __syncwarp();
       staged_seq = c.seq;
+      staged_layer = c.layer;
     }
     const int nrows = min(rpb, c.end - c.i);
     char* kvb = c.kvk ? kv.base[1] : kv.base[0];

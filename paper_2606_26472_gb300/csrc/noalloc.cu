@@ -198,9 +198,10 @@ bool view_ok(const epikv_kv_view* kv, int H, int d, KvDev* out) {
     return true;
   }
   if (kv->layout != EPIKV_LAYOUT_PAGED || !kv->block_table || kv->block_size < 1 || kv->max_blocks_per_seq < 1 ||
-      kv->num_blocks < 1 || kv->stride_block < 0 || kv->stride_block % 8)
+      kv->num_blocks < 1 || kv->stride_block < 0 || kv->stride_block % 8 || kv->stride_table_layer < 0)
     return false;
   out->stride_block = kv->stride_block;
+  out->table_stride_layer = kv->stride_table_layer;
   out->block_table = kv->block_table;
   out->max_blocks = kv->max_blocks_per_seq;
   out->block_size = kv->block_size;

@@ -35,7 +35,7 @@ class epikv_kv_view(C.Structure):
     _fields_ = [("k", C.c_void_p), ("v", C.c_void_p), ("layout", C.c_int32), ("stride_layer", C.c_int64),
                 ("stride_seq", C.c_int64), ("stride_block", C.c_int64), ("stride_token", C.c_int64),
                 ("block_table", C.c_void_p), ("max_blocks_per_seq", C.c_int32), ("block_size", C.c_int32),
-                ("num_blocks", C.c_int32)]
+                ("num_blocks", C.c_int32), ("stride_table_layer", C.c_int64)]
 
 
 class epikv_stats(C.Structure):
@@ -131,9 +131,9 @@ def hidden_view(band_rows, row_stride):
 
 
 def kv_view(k, v, *, layout=EPIKV_LAYOUT_CONTIGUOUS, stride_layer, stride_seq=0, stride_block=0, stride_token,
-            block_table=None, max_blocks_per_seq=0, block_size=0, num_blocks=0):
+            block_table=None, max_blocks_per_seq=0, block_size=0, num_blocks=0, stride_table_layer=0):
     return epikv_kv_view(_ptr(k), _ptr(v), layout, stride_layer, stride_seq, stride_block, stride_token,
-                         _ptr(block_table), max_blocks_per_seq, block_size, num_blocks)
+                         _ptr(block_table), max_blocks_per_seq, block_size, num_blocks, stride_table_layer)
 
 
 # ---------------------------------------------------------------- same names

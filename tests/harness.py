@@ -72,7 +72,7 @@ class Session:
 
     def __init__(self, model, *, n_seq, kinds, layout, max_tokens, max_new, prefill, policies,
                  z_window=64, lag=16, lag_window=64, recency_cap=128, block_size=16, shuffle_blocks=True,
-                 select_chunk=1, layer_budgets=0, device="cuda"):
+                 select_chunk=1, layer_budgets=0, layer_tables=False, device="cuda"):
         self.m = model
         self.n_seq = n_seq
         self.kinds = kinds
@@ -97,12 +97,15 @@ class Session:
         for b in range(n_seq):
             E.epikv_seq_reset(self.ctx, b, self.prefill[b], self.policies[b])
         bt = None
+        self.layer_tables = layer_tables and layout == E.EPIKV_LAYOUT_PAGED
         if layout == E.EPIKV_LAYOUT_PAGED:
             mb = (max_tokens + block_size - 1) // block_size
-            perm = gen.block_permutation(model.seed, n_seq * mb) if shuffle_blocks else np.arange(n_seq * mb)
-            bt = perm.reshape(n_seq, mb)
+            nt = n_seq * mb * (model.num_layers if self.layer_tables else 1)
+            perm = gen.block_permutation(model.seed, nt) if shuffle_blocks else np.arange(nt)
+            bt = perm.reshape(model.num_layers, n_seq, mb) if self.layer_tables else perm.reshape(n_seq, mb)
         self.cache = KVCache(layout, model.num_layers, model.num_kv_heads, model.head_dim, max_seqs=n_seq,
-                             max_tokens=max_tokens, block_size=block_size, block_table=bt, device=device)
+                             max_tokens=max_tokens, block_size=block_size, block_table=bt,
+                             layer_tables=self.layer_tables, device=device)
         self.bt_host = None if bt is None else np.asarray(bt)
         # canary fill: any row the library wrongly writes or reads stands out
         self.cache.k.view(torch.int16).fill_(0x7FC1)
@@ -120,7 +123,8 @@ class Session:
         # cache the new rows are generated into before each layer's copy
         self.n_layer = [[0] * self.L for _ in range(n_seq)]
         self.stage = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, model.num_layers, model.num_kv_heads, model.head_dim,
-                             max_seqs=1, max_tokens=max_new, device=device) if layer_budgets else None
+                             max_seqs=1, max_tokens=max_new, device=device) \
+            if layer_budgets or self.layer_tables else None
 
     # ---------------------------------------------------------------- inputs
     def append(self, entries):
@@ -129,12 +133,13 @@ class Session:
         cu = [0]
         for b, n in entries:
             assert self.n_cache[b] + n <= self.cache.T
-            if self.layer_budgets:
+            if self.stage is not None:   # per-layer slots or per-layer block tables: layer by layer
                 kw = self.stage.synth_kwargs()
                 kw["stride_seq"] = 0
                 self.dt.kv(b, self.n_seen[b], n, 0, self.stage.k, self.stage.v, **kw)
                 for l in range(self.L):
-                    slots = np.arange(self.n_layer[b][l], self.n_layer[b][l] + n)
+                    first = self.n_layer[b][l] if self.layer_budgets else self.n_cache[b]
+                    slots = np.arange(first, first + n)
                     for kind, pool in ((0, self.stage.k), (1, self.stage.v)):
                         self.cache.write_layer_rows(kind, b, l, slots, pool[l, 0, :n], self.bt_host)
             else:

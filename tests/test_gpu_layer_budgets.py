@@ -55,18 +55,21 @@ def _check_layer_bytes(sess, b, layer, positions):
 
 
 CASES = [
-    # layout, kinds, prefill, per-sequence layer budgets (small model: 4 layers), new-token pattern
+    # layout, kinds, prefill, per-sequence layer budgets (small model: 4 layers), new-token pattern,
+    # one block table per layer (a single block pool, stride_layer = 0)
     ("contig_bandz", E.EPIKV_LAYOUT_CONTIGUOUS, BANDZ, (0, 5, 0),
-     ((100, 80, 60, 40), (64, 64, 64, 64), (40, 90, 70, 120)), (7, 1, 33)),
+     ((100, 80, 60, 40), (64, 64, 64, 64), (40, 90, 70, 120)), (7, 1, 33), False),
     ("paged_lag", E.EPIKV_LAYOUT_PAGED, LAGKV, (0, 3, 20),
-     ((48, 96, 72, 120), (130, 30, 30, 130), (60, 61, 62, 63)), (16, 5, 40)),
+     ((48, 96, 72, 120), (130, 30, 30, 130), (60, 61, 62, 63)), (16, 5, 40), False),
     ("paged_both", E.EPIKV_LAYOUT_PAGED, BANDZ | LAGKV, (3, 0, 0),
-     ((80, 50, 110, 20), (33, 66, 99, 132), (90, 90, 45, 45)), (1, 9, 64)),
+     ((80, 50, 110, 20), (33, 66, 99, 132), (90, 90, 45, 45)), (1, 9, 64), False),
+    ("paged_both_layer_tables", E.EPIKV_LAYOUT_PAGED, BANDZ | LAGKV, (0, 4, 0),
+     ((120, 90, 60, 30), (50, 100, 50, 100), (77, 66, 55, 44)), (5, 16, 33), True),
 ]
 
 
-@pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks", CASES, ids=[c[0] for c in CASES])
-def test_layer_budget_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chunks):
+@pytest.mark.parametrize("name,layout,kinds,prefill,budgets,chunks,layer_tables", CASES, ids=[c[0] for c in CASES])
+def test_layer_budget_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chunks, layer_tables):
     model = W.small_model(2000 + len(name))
     n_seq, L = 3, model.num_layers
     lengths = (301, 260, 333)
@@ -75,7 +78,7 @@ def test_layer_budget_decode_parity_small(gpu_lib, name, layout, kinds, prefill,
     max_new = max(chunks)
     T_cap = max(max(k) for k in budgets) + slack + max_new + 1
     sess = Session(model, n_seq=n_seq, kinds=kinds, layout=layout, max_tokens=T_cap, max_new=max_new,
-                   prefill=prefill, policies=policies, layer_budgets=1)
+                   prefill=prefill, policies=policies, layer_budgets=1, layer_tables=layer_tables)
     refs = [OracleTrace(model, sess.dt.tabs, b, lengths[b], kinds) for b in range(n_seq)]
     triggers = [max(budgets[b]) + slack for b in range(n_seq)]
     replay = [LayerReplay(L, budgets[b], prefill[b], triggers[b]) for b in range(n_seq)]
@@ -146,6 +149,37 @@ def test_equal_layer_budgets_are_the_token_path_bit_for_bit(gpu_lib):
         np.testing.assert_array_equal(np.stack(a.cache_rows_u16(s, np.arange(n))),
                                       np.stack(b.cache_rows_u16(s, np.arange(n))))
     assert E.epikv_get_stats(a.ctx)["layer_rows_moved"] == E.epikv_get_stats(b.ctx)["layer_rows_moved"] > 0
+    assert a.error() == b.error() == (E.EPIKV_OK, 0)
+    a.close()
+    b.close()
+
+
+def test_token_budgets_over_per_layer_block_tables_equal_the_shared_table(gpu_lib):
+    """One block pool with a block table per layer (stride_layer = 0) holds
+    the same rows as the layer-plane layout with one shared table, and the
+    scores, selections and compacted rows are the same bit for bit."""
+    model = W.small_model(66)
+    kw = dict(n_seq=3, kinds=BANDZ | LAGKV, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=150, max_new=24,
+              prefill=(0, 2, 0), policies=(BANDZ, LAGKV, LAGKV))
+    a, b = Session(model, layer_tables=True, **kw), Session(model, **kw)
+    assert a.kv.stride_layer == 0 and a.kv.stride_table_layer > 0
+    budgets, triggers = [90, 64, 110], [100, 70, 125]
+    for step in range(24):
+        entries = [(s, (24, 3, 11)[(s + step) % 3]) for s in range(3)]
+        a.step(entries, budgets, triggers)
+        b.step(entries, budgets, triggers)
+        for s in range(3):
+            assert a.n_cache[s] == b.n_cache[s]
+            for kind in (BANDZ, LAGKV):
+                pa, sa = a.read(s, kind)
+                pb, sb = b.read(s, kind)
+                np.testing.assert_array_equal(pa, pb)
+                np.testing.assert_array_equal(sa.view(np.uint32), sb.view(np.uint32))
+    for s in range(3):
+        n = a.n_cache[s]
+        np.testing.assert_array_equal(np.stack(a.cache_rows_u16(s, np.arange(n))),
+                                      np.stack(b.cache_rows_u16(s, np.arange(n))))
+    assert E.epikv_get_stats(a.ctx)["evictions"] > 20
     assert a.error() == b.error() == (E.EPIKV_OK, 0)
     a.close()
     b.close()
