@@ -656,13 +656,16 @@ def run_pertoken(args):
 def run_layers32k(args):
     """Per-layer budgets on the 32 x 32k Lag-KV paged workload: layer l of
     every sequence keeps its own budget K_l (a pyramid from 1.5 K at layer 0
-    to 0.5 K at the last layer, mean K) and every step evicts every layer
-    (trigger K_max + C - 1).  One step = C new tokens per sequence: scoring,
-    the per-layer selection and the per-layer compaction (epikv_step).  Each
-    step's new K/V rows go to every layer's own next slots, which depend on
-    the previous step, so they are written between steps, untimed (in a
-    decode loop the model's forward writes them); the time is the sum of the
-    steps' device times (CUDA events on the launching stream)."""
+    to 0.5 K at the last layer, mean K) in its own blocks of one shared pool
+    (a block table per layer), so a layer holds at most K_l + C tokens and
+    the pool is sized by the budgets.  Every step evicts every layer that is
+    over its budget (trigger K_min + C - 1).  One step = C new tokens per
+    sequence: scoring, the per-layer selection and the per-layer compaction
+    (epikv_step).  Each step's new K/V rows go to every layer's own next
+    slots, which depend on the previous step, so they are written between
+    steps, untimed (in a decode loop the model's forward writes them); the
+    time is the sum of the steps' device times (CUDA events on the launching
+    stream).  The caches are filled by the same steps, untimed."""
     import torch
 
     from paper_2606_26472_gb300 import build as B
@@ -684,14 +687,21 @@ def run_layers32k(args):
     L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
     bs = wl.block_size
     budgets = W.pyramid_budgets(K, L)
-    K_max = max(budgets)
+    K_max, K_min = max(budgets), min(budgets)
     T_cap = K_max + C
-    assert T_cap % bs == 0
+    assert T_cap % bs == 0 and C % bs == 0 and all(k % bs == 0 for k in budgets)
     mb = T_cap // bs
-    n_blocks = Bn * mb
-    perm = gen.block_permutation(m.seed, n_blocks).reshape(Bn, mb)
+    need = [(k + C) // bs for k in budgets]           # blocks a layer of a sequence ever holds
+    n_blocks = Bn * sum(need)
+    perm = gen.block_permutation(m.seed, n_blocks)
+    tab = np.full((L, Bn, mb), -1, np.int32)
+    o = 0
+    for l in range(L):
+        for b in range(Bn):
+            tab[l, b, :need[l]] = perm[o:o + need[l]]
+            o += need[l]
     cache = KVCache(E.EPIKV_LAYOUT_PAGED, L, H, d, max_seqs=Bn, max_tokens=T_cap, block_size=bs,
-                    num_blocks=n_blocks, block_table=perm, device=dev)
+                    num_blocks=n_blocks, block_table=tab, layer_tables=True, device=dev)
     view = cache.view()
     stage = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, L, H, d, max_seqs=Bn, max_tokens=C, device=dev)
     dt = DeviceTrace(m, dev)
@@ -705,29 +715,25 @@ def run_layers32k(args):
         E.epikv_seq_reset(ctx, b, 0, E.EPIKV_SCORE_LAGKV)
     seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
     cu_new = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * C).contiguous()
-    # the first K_fill tokens of every trace, in every layer, scored C at a time (no eviction yet)
-    K_fill = K_max // C * C
-    for b in range(Bn):
-        dt.kv(b, 0, K_fill, 0, cache.k, cache.v, **cache.synth_kwargs())
-    for _ in range(K_fill // C):
-        E.epikv_score_update(ctx, Bn, seq_ids, cu_new, C, None, view)
     budget = torch.tensor([list(budgets)] * Bn, dtype=torch.int32, device=dev)
-    trigger = torch.full((Bn,), K_max + C - 1, dtype=torch.int32, device=dev)
+    trigger = torch.full((Bn,), K_min + C - 1, dtype=torch.int32, device=dev)
     n_out = torch.empty((Bn, L), dtype=torch.int32, device=dev)
-    n_layer = np.full((Bn, L), K_fill, dtype=np.int64)
+    n_layer = np.zeros((Bn, L), dtype=np.int64)
     rows = np.arange(Bn)[:, None]
 
     def write_new(pos0):   # step's new rows into every layer's next C slots
         for b in range(Bn):
-            dt.kv(b, pos0, C, 0, stage.k, stage.v, **stage.synth_kwargs())
+            dt.kv(b, pos0, C, 0, stage.k, stage.v, **dict(stage.synth_kwargs(), stride_seq=C * H * d))
         for l in range(L):
             slots = n_layer[:, l:l + 1] + np.arange(C)
-            flat = perm[rows, slots // bs] * bs + slots % bs
+            flat = tab[l][rows, slots // bs] * bs + slots % bs
             idx = torch.as_tensor(flat.reshape(-1), device=dev)
-            cache.k[l].view(-1, H, d)[idx] = stage.k[l].reshape(-1, H, d)
-            cache.v[l].view(-1, H, d)[idx] = stage.v[l].reshape(-1, H, d)
+            cache.k.view(-1, H, d)[idx] = stage.k[l].reshape(-1, H, d)
+            cache.v.view(-1, H, d)[idx] = stage.v[l].reshape(-1, H, d)
 
-    n_steps = args.warmup + args.steps
+    fill = K_max // C                                   # steps until every layer has reached its budget
+    n_steps = fill + args.warmup + args.steps
+    t0 = fill + args.warmup
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_steps)]
     phase = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_steps)]
     for e in (x for p in phase for x in p):
@@ -740,17 +746,18 @@ def run_layers32k(args):
     clocks = None
     stats0 = None
     for st in range(n_steps):
-        if st == args.warmup:
+        if st == t0:
             torch.cuda.synchronize()
             stats0 = E.epikv_get_stats(ctx)
             clocks = Clocks(gpu_id)
             clocks.start()
-        write_new(K_fill + st * C)
+        write_new(st * C)
         E.epikv_set_phase_events(ctx, phase[st])
         ev[st][0].record(stream)
         E.epikv_step(ctx, Bn, seq_ids, cu_new, C, budget, trigger, None, view, n_out)
         ev[st][1].record(stream)
         n_layer = n_out.cpu().numpy().astype(np.int64)
+        assert (n_layer <= np.asarray(budgets)[None, :] + C).all()
     torch.cuda.synchronize()
     clk = clocks.stop()
     E.epikv_set_phase_events(ctx, None)
@@ -758,7 +765,7 @@ def run_layers32k(args):
     assert st_ == E.EPIKV_OK, f"device error {code}"
     assert (n_layer == np.asarray(budgets)[None, :]).all()
     stats1 = E.epikv_get_stats(ctx)
-    timed = range(args.warmup, n_steps)
+    timed = range(t0, n_steps)
     ms = sum(ev[i][0].elapsed_time(ev[i][1]) for i in timed)
     t_score = sum(phase[i][0].elapsed_time(phase[i][1]) for i in timed)
     t_select = sum(phase[i][1].elapsed_time(phase[i][2]) for i in timed)
@@ -769,6 +776,7 @@ def run_layers32k(args):
     compact_bytes = 2 * layer_rows * 2 * H * d * 2          # read + write of K and V rows of one layer
     peak, peak_src = measured_hbm_peak()
     ach = compact_bytes / (t_compact / 1e3) / 1e9
+    block_bytes = 2 * bs * H * d * 2                        # K and V of one block
     line = {
         "metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
@@ -776,8 +784,10 @@ def run_layers32k(args):
         "config": {"workload": f"batch{Bn}_32k_lagkv_paged16_layerbudgets_pyramid_mean{K}_chunk{C}",
                    "sequences": Bn, "layers": L, "kv_heads": H, "head_dim": d, "chunk": C,
                    "layer_budgets": [budgets[0], budgets[-1]], "budget_mean": K, "score": "lagkv_lag16_w64",
+                   "pool": "one block pool, a block table per layer: %.1f GiB (one table for all layers: %.1f GiB)"
+                           % (n_blocks * block_bytes / 2 ** 30, Bn * mb * L * block_bytes / 2 ** 30),
                    "timing": "sum of per-step device times; each step's new K/V written before it, untimed",
-                   "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
+                   "l2": "inputs larger than L2"},
         "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
                                 "compact": t_compact / args.steps},
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
