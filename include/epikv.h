@@ -21,8 +21,10 @@
  *   - Ownership: the caller owns every buffer (the workspace, hidden rows,
  *     the K/V pool, block tables, outputs).  The library never allocates
  *     device memory; epikv_init allocates only its small host-side context.
- *   - Asynchrony: every call except epikv_get_error, epikv_get_stats and
- *     epikv_read_slots only enqueues work on the given stream and returns.
+ *   - Asynchrony: every call except epikv_get_error, epikv_get_stats,
+ *     epikv_read_slots and epikv_read_layer_slots only enqueues work on the
+ *     given stream and returns (no synchronisation, no allocation), so a
+ *     whole decode step can be captured once in a CUDA graph and replayed.
  *     Calls on one context must be ordered on one stream.
  *   - Host validation failures return EPIKV_EINVAL and enqueue nothing.
  *   - Device-side anomalies (an index out of range, a batch larger than

@@ -29,9 +29,9 @@
 // slots (the union of all layers) with a 64-bit mask per slot of the layers
 // holding it.  layer_keep_kernel (a CTA per layer and sequence) finds layer
 // l's threshold of M_l = K_l - P - R over the union's candidates, writes the
-// layer's kept list in its own slot numbering and a keep byte per union slot;
-// layer_union_kernel (a CTA per sequence) turns the keep bytes into the new
-// masks and compacts the union's metadata.
+// layer's kept list in its own slot numbering and a keep bit per union slot
+// (a 32-bit word per 32 slots); layer_union_kernel (a CTA per sequence) turns
+// the keep bits into the new masks and compacts the union's metadata.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -425,7 +425,7 @@ __global__ void __launch_bounds__(kLayerThreads) layer_keep_kernel(DevState st, 
   int n_eq, n_old;
   int q = warp_base<NW>(ceq, &n_eq, wt);
   const int old_base = warp_base<NW>(cold, &n_old, wt);
-  // pass 2: the layer's decision per slot (a keep byte), per-warp kept counts
+  // pass 2: the layer's decision per slot (a keep bit, one word per 32 slots), per-warp kept counts
   int cnew = 0;
   for (int i0 = sg.lo; i0 < sg.hi; i0 += 32) {
     const int i = i0 + lane;
@@ -480,7 +480,7 @@ __global__ void __launch_bounds__(kLayerThreads) layer_keep_kernel(DevState st, 
 }
 
 // The union of the layers after a per-layer selection, one CTA per batch
-// entry: each slot's new layer mask (from the keep bytes), the kept slots of
+// entry: each slot's new layer mask (from the keep bits), the kept slots of
 // the union (the largest layer's), and the in-place compaction of the slot
 // metadata (scores, positions, masks).
 __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, Dims dm,
