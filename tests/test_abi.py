@@ -52,6 +52,13 @@ def test_workspace_sizing_and_invalid_configs(lib):
     # chunk-level selection adds one key per slot; 0 and 1 are the token rule
     assert E.epikv_workspace_bytes(cfg(select_chunk=0)) == E.epikv_workspace_bytes(cfg(select_chunk=1)) == ok
     assert E.epikv_workspace_bytes(cfg(select_chunk=16)) >= ok + 4 * 4 * 1024
+    # per-layer budgets: per-layer lengths, masks, keep bits and kept lists
+    lay = E.epikv_workspace_bytes(cfg(layer_budgets=1))
+    assert lay >= ok + 4 * 1024 * (8 + 8 + 4 + 4 * 31)
+    for bad in (dict(layer_budgets=2), dict(layer_budgets=1, num_layers=65),
+                dict(layer_budgets=1, select_chunk=8)):
+        assert E.epikv_workspace_bytes(cfg(**bad)) == 0, bad
+    assert E.epikv_workspace_bytes(cfg(layer_budgets=1, num_layers=64)) > 0
     for bad in (dict(max_seqs=0), dict(head_dim=96), dict(head_dim=4), dict(hidden=4100), dict(n_band_a=0),
                 dict(z_window=0), dict(score_kinds=0), dict(score_kinds=64), dict(num_kv_heads=64),
                 dict(max_new_tokens=0), dict(z_window=2000), dict(score_kinds=2, lag=0),

@@ -93,3 +93,34 @@ def test_kept_list_that_is_not_increasing(gpu_lib):
     E.epikv_compact(sess.ctx, 2, ids, bad, 64, sess.kv)
     assert sess.error() == (E.EPIKV_EDEVICE, E.EPIKV_DEV_KEPT)
     sess.close()
+
+
+def test_negative_layer_table_stride_is_rejected_on_the_host(gpu_lib):
+    sess = _session(kinds=E.EPIKV_SCORE_LAGKV)
+    seq_ids, cu, mx, hv = sess.append([(0, 8)])
+    view = sess.cache.view()
+    view.stride_table_layer = -1
+    with pytest.raises(E.EpikvError) as err:
+        E.epikv_score_update(sess.ctx, 1, seq_ids, cu, mx, hv, view)
+    assert err.value.status == E.EPIKV_EINVAL
+    assert sess.error() == (E.EPIKV_OK, 0)                        # nothing was enqueued
+    sess.close()
+
+
+def test_layer_budgets_that_break_the_nesting_are_reported(gpu_lib):
+    """Per-layer budgets must stay fixed for a sequence: after layer 1 was cut
+    to 20 tokens, giving it the largest budget asks it to keep tokens it no
+    longer holds, which the selection reports instead of inventing rows."""
+    model = W.small_model(32)
+    sess = Session(model, n_seq=1, kinds=E.EPIKV_SCORE_BANDZ, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=96,
+                   max_new=48, prefill=(0,), policies=(E.EPIKV_SCORE_BANDZ,), layer_budgets=1)
+    sess.score_update([(0, 48)])
+    sess.select([0], [[40, 20, 40, 40]])
+    sess.compact([0])
+    assert sess.error() == (E.EPIKV_OK, 0) and sess.n_layer[0] == [40, 20, 40, 40]
+    sess.score_update([(0, 16)])
+    sess.select([0], [[20, 40, 40, 40]])
+    sess.compact([0])
+    assert sess.error() == (E.EPIKV_EDEVICE, E.EPIKV_DEV_KEPT)
+    assert sess.n_layer[0][1] <= 36                                # layer 1 kept only rows it holds
+    sess.close()
