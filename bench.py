@@ -50,7 +50,11 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    p.add_argument("--e2e-steps", type=int, default=20)
+    # host-to-device copies share the machine's host memory path: over ~1 s a
+    # burst of slow copies on the shared host costs a few percent, not half
+    p.add_argument("--e2e-steps", type=int, default=100)
+    # CTAs of the end-to-end measurement's host-to-device upload kernel
+    p.add_argument("--upload-ctas", type=int, default=32)
     # a scaled-down variant of the same workload, for profiler captures
     p.add_argument("--sequences", type=int, default=32)
     p.add_argument("--budget", type=int, default=8192)
@@ -384,19 +388,29 @@ def run_ours(args):
             payload[j, 1].copy_(cache.v[:, lo:lo + Bn * fresh])
         lens = torch.empty((e2e_steps, Bn), dtype=torch.int32, pin_memory=True)
         copy_stream = torch.cuda.Stream(device=dev)
-        copied = [torch.cuda.Event() for _ in range(e2e_steps)]
-        stepped = [torch.cuda.Event() for _ in range(e2e_steps)]
+        copied = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+        stepped = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+        copy_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+        step_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+
+        # one strided upload per K and V and step (32 layer planes of 8 MiB
+        # each), read from the pinned host buffer by SM loads over the host
+        # link: the copy engines of this platform stall every ~0.5 s for
+        # ~0.1 s, the SM path does not (both move ~210 GB/s otherwise)
+        from synth.device import upload_2d
+        plane = Bn * fresh * bs * H * d * 2                 # bytes of one layer's new rows
+        pitch = cache.k.stride(0) * 2                       # bytes between layer planes of the pool
+        up_ctas = args.upload_ctas
 
         def h2d(i):   # step i's new K/V into block set i % 2, after step i-2 released it
             lo_i = e2e_base + (i % 2) * Bn * fresh
-            with torch.cuda.stream(copy_stream):
-                if i >= 2:
-                    copy_stream.wait_event(stepped[i - 2])
-                src = payload[i % n_payload]
-                for kind, pool in ((0, cache.k), (1, cache.v)):
-                    for l in range(L):
-                        pool[l, lo_i:lo_i + Bn * fresh].copy_(src[kind, l], non_blocking=True)
-                copied[i].record(copy_stream)
+            if i >= 2:
+                copy_stream.wait_event(stepped[i - 2])
+            copy_start[i].record(copy_stream)
+            src = payload[i % n_payload]
+            for kind, pool in ((0, cache.k), (1, cache.v)):
+                upload_2d(pool[0, lo_i].data_ptr(), pitch, src[kind].data_ptr(), plane, plane, L, up_ctas, copy_stream)
+            copied[i].record(copy_stream)
 
         torch.cuda.synchronize()
         if world > 1:
@@ -410,6 +424,7 @@ def run_ours(args):
             if i + 1 < e2e_steps:
                 h2d(i + 1)
             stream.wait_event(copied[i])
+            step_start[i].record(stream)
             step(None, views_e[i % 2])
             stepped[i].record(stream)
             lens[i].copy_(n_out, non_blocking=True)
@@ -417,9 +432,17 @@ def run_ours(args):
         torch.cuda.synchronize()
         e_ms, e_value = aggregate_ranks(e0.elapsed_time(e1), Bn * C * e2e_steps, world, dev)
         assert (lens.numpy() == K).all()
+        copy_ms = sorted(copy_start[i].elapsed_time(copied[i]) for i in range(e2e_steps))
+        step_ms = sorted(step_start[i].elapsed_time(stepped[i]) for i in range(e2e_steps))
         e2e = {"value": e_value, "unit": UNIT,
                "h2d_bytes_per_step": int(payload[0].numel() * 2), "d2h_bytes_per_step": Bn * 4,
-               "steps": e2e_steps, "overlap": "step i+1's host-to-device copy runs on a side stream during step i"}
+               "steps": e2e_steps,
+               "overlap": "step i+1's host-to-device upload (SM loads of pinned host memory) runs on a side stream "
+                          "during step i",
+               "median_ms": {"h2d_copy": copy_ms[len(copy_ms) // 2], "step": step_ms[len(step_ms) // 2],
+                             "wall_per_step": e_ms / e2e_steps},
+               "max_ms": {"h2d_copy": copy_ms[-1], "step": step_ms[-1]},
+               "slow_copies": sum(c > 2 * copy_ms[len(copy_ms) // 2] for c in copy_ms)}
         st_, code = E.epikv_get_error(ctx)
         assert st_ == E.EPIKV_OK, f"device error {code} in e2e"
 

@@ -37,8 +37,19 @@ def load():
                                        C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int,
                                        C.c_int64, C.c_int64, C.c_int64, C.c_int64, C.c_void_p, C.c_int, C.c_int,
                                        C.c_void_p]
+        lib.synth_upload_2d.restype = C.c_int
+        lib.synth_upload_2d.argtypes = [C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_size_t, C.c_size_t,
+                                        C.c_int, C.c_void_p]
         _lib = lib
     return _lib
+
+
+def upload_2d(dst, dpitch, src, spitch, width, height, ctas, stream=None):
+    """Host-to-device copy of `height` rows of `width` bytes by SM loads of
+    pinned host memory (see synth_upload_2d)."""
+    r = load().synth_upload_2d(dst, dpitch, src, spitch, width, height, ctas, _stream(stream))
+    if r != 0:
+        raise RuntimeError(f"synth_upload_2d failed ({r})")
 
 
 def _stream(stream):

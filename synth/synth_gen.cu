@@ -189,9 +189,35 @@ __global__ void kv_batch_kernel(uint64_t seed, int n, const int32_t* __restrict_
   *reinterpret_cast<uint4*>(vw.base[kind] + (row + h * d + j0) * 2) = q;
 }
 
+// Delivery of host-resident inputs: row r (of gridDim.y) of `width16` 16-byte
+// vectors, read from pinned host memory through unified addressing by the SMs
+// (no copy engine) and stored to device memory.
+__global__ void upload_kernel(char* __restrict__ dst, size_t dpitch, const char* __restrict__ src, size_t spitch,
+                              size_t width16) {
+  const size_t r = blockIdx.y;
+  for (size_t c = blockIdx.x * (size_t)blockDim.x + threadIdx.x; c < width16; c += (size_t)gridDim.x * blockDim.x)
+    *reinterpret_cast<uint4*>(dst + r * dpitch + c * 16) = *reinterpret_cast<const uint4*>(src + r * spitch + c * 16);
+}
+
 }  // namespace
 
 extern "C" {
+
+// `height` rows of `width` bytes from pinned host memory (rows `spitch` apart)
+// to device memory (rows `dpitch` apart), read by about `ctas` CTAs of SM
+// loads over the host link: the host-to-device input delivery of the
+// end-to-end measurement.  Pointers, pitches and width are 16-byte multiples.
+int synth_upload_2d(void* dst, size_t dpitch, const void* src, size_t spitch, size_t width, size_t height, int ctas,
+                    cudaStream_t stream) {
+  if (!dst || !src || ctas < 1 || (width & 15) || (dpitch & 15) || (spitch & 15) || ((uintptr_t)dst & 15) ||
+      ((uintptr_t)src & 15) || width > dpitch || width > spitch || height > 65535)
+    return 1;
+  if (width == 0 || height == 0) return 0;
+  const int gx = ctas / (int)height > 0 ? ctas / (int)height : 1;
+  upload_kernel<<<dim3(gx, (unsigned)height), 512, 0, stream>>>(static_cast<char*>(dst), dpitch,
+                                                                static_cast<const char*>(src), spitch, width / 16);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
 
 // Rows [n][D] of one hidden layer for positions pos0..pos0+n-1 of one sequence.
 int synth_hidden(uint64_t seed, int seq, int layer, int pos0, int n, int D, float scale, float drift, float seg_amp,
