@@ -672,7 +672,7 @@ def run_pertoken(args):
                        "l2": "band rows of every token resident, %.1f GiB" % (hid.numel() * 2 / 2 ** 30)},
             "per_token_us": {"graph": 1e3 * ms_graph / (args.steps * G), "eager": 1e3 * ms_eager / (args.steps * G)},
             "eager_value": tokens / (ms_eager / 1e3),
-            "gpu_launches": 2 * G * args.steps}
+            "gpu_launches": G * args.steps}   # one fused g + z launch per decode step
     print(json.dumps(line), flush=True)
 
 

@@ -606,6 +606,145 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
   }
 }
 
+
+// One new token per sequence with the band kinds only (a decode step):
+// g and the rolling z-score in one launch.  grid (band layers, batch
+// entries), kGThreads threads: each CTA forms its band row's g exactly as
+// bandz_g_kernel does (same per-thread vectors, warp sums and fixed-order
+// cross-warp sum) and writes the ring and h_prev; the last CTA of a sequence
+// (atomic ticket after a fence; no CTA waits) stages every band's window from
+// the ring in shared memory -- the earlier positions' g are the per-sequence
+// running state -- and forms z and the score exactly as score_finalize_kernel
+// does (a lane per band, the same shifted two-pass, the same butterfly over
+// the lanes), then commits the sequence's counters.  Results equal the
+// two-kernel path bit for bit.
+template <int VPT>
+__global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dims dm, BandRows rows,
+                                                                 int64_t row_stride,
+                                                                 const int32_t* __restrict__ seq_ids,
+                                                                 const int32_t* __restrict__ cu_new) {
+  const int band = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int seq = seq_ids[b];
+  const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > 1 || cu_new[0] != 0) {
+    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  if (n_new == 0) return;
+  const int nb = dm.nA + dm.nB;
+  const int nc0 = st.n_cache[seq];
+  const int pos = st.n_seen[seq];
+  if (nc0 + 1 > dm.T) {
+    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+    return;
+  }
+  const int par = st.hp_parity[seq];
+  const int VR = dm.D >> 3;
+  const int Gm = dm.G - 1;
+  __shared__ float red[kGThreads / 32];
+  __shared__ int s_last;
+
+  // ---- g of this band layer (the row against the previous one, h_prev)
+  const __nv_bfloat16* cur = rows.p[band] + (int64_t)r0 * row_stride;
+  const __nv_bfloat16* prow = st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D;
+  __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
+  uint4 c[VPT], p[VPT];
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int v = tid + k * kGThreads;
+    c[k] = v < VR ? ld_stream16(cur + v * 8) : make_uint4(0, 0, 0, 0);
+    p[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
+  }
+  float acc = 0.f;
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    float cf[8], pf[8];
+    unpack8(c[k], cf);
+    unpack8(p[k], pf);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float dlt = cf[e] - pf[e];
+      acc = fmaf(dlt, dlt, acc);
+    }
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) red[warp] = acc;
+#pragma unroll
+  for (int k = 0; k < VPT; ++k) {
+    const int v = tid + k * kGThreads;
+    if (v < VR) *reinterpret_cast<uint4*>(hp_wr + v * 8) = c[k];
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kGThreads / 32; ++w) sum += red[w];
+    if (pos >= 1) st.g_ring[((size_t)seq * nb + band) * dm.G + (pos & Gm)] = sqrtf(sum);
+    __threadfence();
+    s_last = atomicAdd(&st.ticket[seq], 1u) == (unsigned)(nb - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+
+  // ---- the last CTA of the sequence: z of every band, the score, the commit
+  __threadfence();
+  extern __shared__ float win[];  // [nb][w]: win[band * w + k] = g at position pos - k
+  const int w = dm.z_window;
+  const int n = pos >= 1 ? min(w, pos) : 0;
+  for (int idx = tid; idx < nb * n; idx += kGThreads) {
+    const int bb = idx / n, k = idx - bb * n;
+    win[bb * w + k] = __ldcg(st.g_ring + ((size_t)seq * nb + bb) * dm.G + ((pos - k) & Gm));
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int lpt = nb <= 16 ? 16 : 32;  // the lanes of one token, as in score_finalize_kernel
+    const int bl = lane % lpt;
+    const bool live = lane < lpt && pos >= 1 && bl < nb;
+    float za = 0.f, zb = 0.f, ma = 0.f, mb = 0.f;
+    if (live) {
+      const float* row = win + bl * w;  // row[k] = g at position pos - k
+      if (dm.kinds & EPIKV_SCORE_BANDZ) {
+        const float gnew = row[0];
+        float dsum = 0.f;
+        for (int k = 0; k < n; ++k) dsum += row[k] - gnew;
+        const float mean_d = dsum / (float)n;
+        float dev = 0.f;
+        for (int k = 0; k < n; ++k) {
+          const float e = (row[k] - gnew) - mean_d;
+          dev = fmaf(e, e, dev);
+        }
+        const float sigma = sqrtf(dev / (float)n);
+        const float z = -mean_d / (sigma + dm.z_eps);
+        if (bl < dm.nA) za = z; else zb = z;
+      }
+      if (dm.kinds & EPIKV_SCORE_HSVAR) {
+        float sum = 0.f;
+        for (int k = 0; k < n; ++k) sum += row[k];
+        const float gbar = sum / (float)n;
+        if (bl < dm.nA) ma = gbar; else mb = gbar;
+      }
+    }
+    for (int o = lpt >> 1; o > 0; o >>= 1) {
+      za += __shfl_xor_sync(0xffffffffu, za, o);
+      zb += __shfl_xor_sync(0xffffffffu, zb, o);
+      ma += __shfl_xor_sync(0xffffffffu, ma, o);
+      mb += __shfl_xor_sync(0xffffffffu, mb, o);
+    }
+    if (lane == 0) {
+      const size_t slot = (size_t)seq * dm.T + nc0;
+      st.pos[slot] = pos;
+      if (dm.kinds & EPIKV_SCORE_BANDZ) st.score[0][slot] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
+      if (dm.kinds & EPIKV_SCORE_HSVAR) st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
+      st.n_cache[seq] = nc0 + 1;
+      st.n_seen[seq] = pos + 1;
+      st.hp_parity[seq] = par ^ 1;
+      atomicAdd(&st.stats[0], 1ull);
+      st.ticket[seq] = 0u;
+    }
+  }
+}
+
 // ------------------------------------------------------------------ launchers
 // dynamic shared memory of the finalize kernel: the band windows of a tile
 static size_t finalize_smem(const Dims& dm) {
@@ -615,7 +754,11 @@ static size_t finalize_smem(const Dims& dm) {
 
 cudaError_t finalize_prepare() {
   const int mx = (int)((size_t)kMaxBand * (kFinTile + kMaxWindow - 1) * sizeof(float));
-  cudaError_t e = cudaFuncSetAttribute(score_finalize_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  const int wmx = (int)((size_t)kMaxBand * kMaxWindow * sizeof(float));
+  cudaError_t e = cudaFuncSetAttribute(bandz_token_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
@@ -627,6 +770,22 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
                                 const KvDev* kv, int num_sms, cudaStream_t stream, int* launches) {
   if (n_seq == 0 || max_new == 0) return cudaSuccess;
   const int nb = dm.nA + dm.nB;
+  if (max_new == 1 && !(dm.kinds & kKvKinds)) {  // a decode step of the band kinds: one fused launch
+    BandRows rows;
+    for (int i = 0; i < kMaxBand; ++i)
+      rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
+    const int vr = dm.D / 8;
+    const dim3 grid(nb, n_seq);
+    const size_t wsm = (size_t)nb * dm.z_window * sizeof(float);  // the last CTA's staged windows
+    if (vr <= kGThreads)
+      bandz_token_kernel<1><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
+    else if (vr <= 2 * kGThreads)
+      bandz_token_kernel<2><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
+    else
+      bandz_token_kernel<4><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
+    ++*launches;
+    return cudaGetLastError();
+  }
   if (dm.kinds & kBandKinds) {
     BandRows rows;
     for (int i = 0; i < kMaxBand; ++i)
