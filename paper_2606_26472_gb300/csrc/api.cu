@@ -206,6 +206,7 @@ epikv_status epikv_init(epikv_ctx** out, const epikv_config* cfg, void* d_worksp
   int per_sm = 1;
   if (e == cudaSuccess) e = compact_prepare(ctx->device, &per_sm);
   if (e == cudaSuccess) e = finalize_prepare();
+  if (e == cudaSuccess) e = select_prepare();
   ctx->compact_ctas = ctx->num_sms * per_sm;
   if (e == cudaSuccess) e = cudaMemsetAsync(d_workspace, 0, need, stream);
   if (e == cudaSuccess) e = launch_init_state(ctx->st, ctx->dm, stream);

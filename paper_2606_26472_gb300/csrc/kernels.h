@@ -22,6 +22,7 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm);
 cudaError_t finalize_prepare();
+cudaError_t select_prepare();
 
 cudaError_t launch_reset_seq(const DevState& st, const Dims& dm, int seq, int prefill, int policy,
                              cudaStream_t stream);

@@ -8,7 +8,9 @@
 // candidates equal to it the lowest slots are kept.  Two block-wide ordered
 // scans emit the kept list in ascending slot order.  The slot metadata
 // (scores of every kind and positions) is then compacted in place, which is
-// safe in increasing order because kept[i] >= i.
+// safe in increasing order because kept[i] >= i.  When the cache has at most
+// kSelStagedMax slots the candidates' keys are first staged in shared memory,
+// and the radix passes and scans read them there.
 //
 // Chunk-level selection (select_chunk = C > 1; the paper names chunk-level
 // scoring as future work, Sec. 5): a first pass gives every candidate slot the
@@ -162,7 +164,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
                                                              const int32_t* __restrict__ budget,
                                                              const int32_t* __restrict__ trigger,
                                                              int32_t* __restrict__ kept_out, int kept_stride,
-                                                             int32_t* __restrict__ n_kept_out) {
+                                                             int32_t* __restrict__ n_kept_out, int staged_cap) {
   const int b = blockIdx.x, tid = threadIdx.x;
   const int seq = seq_ids[b];
   if (seq < 0 || seq >= dm.S) {
@@ -218,7 +220,18 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
     }
     __syncthreads();
   }
-  auto key_at = [&](int i) -> uint32_t { return kChunked ? ck[i] : order_key(sc[i]); };
+  // the candidates' keys staged in shared memory when the launch provided room
+  // for the cache (every later pass reads them there instead of from L2)
+  extern __shared__ uint32_t skey[];
+  const bool staged = staged_cap >= c1 - c0;
+  if (staged) {
+    for (int i = c0 + tid; i < c1; i += kSelThreads) skey[i - c0] = kChunked ? ck[i] : order_key(sc[i]);
+    __syncthreads();
+  }
+  auto key_at = [&](int i) -> uint32_t {
+    if (staged) return skey[i - c0];
+    return kChunked ? ck[i] : order_key(sc[i]);
+  };
 
   __shared__ RadixShared rs;
   __shared__ int sh_scan[32];
@@ -574,6 +587,18 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
   }
 }
 
+// Candidate keys staged in shared memory: caches of up to kSelStagedMax slots.
+constexpr int kSelStagedMax = 48 * 1024;  // 192 KiB of u32 keys
+static int sel_staged_cap(const Dims& dm) { return dm.T <= kSelStagedMax ? dm.T : 0; }
+static size_t sel_smem(const Dims& dm) { return (size_t)sel_staged_cap(dm) * sizeof(uint32_t); }
+
+cudaError_t select_prepare() {
+  const int mx = kSelStagedMax * (int)sizeof(uint32_t);
+  cudaError_t e = cudaFuncSetAttribute(select_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  return e;
+}
+
 cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
                           const int32_t* budget, const int32_t* trigger, int32_t* kept, int kept_stride,
                           int32_t* n_kept, cudaStream_t stream, int* launches) {
@@ -586,11 +611,11 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
     ++*launches;
     layer_union_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept_stride);
   } else if (dm.select_chunk > 1)
-    select_kernel<true><<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
-                                                           n_kept);
+    select_kernel<true><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
+                                                                      kept_stride, n_kept, sel_staged_cap(dm));
   else
-    select_kernel<false><<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept, kept_stride,
-                                                            n_kept);
+    select_kernel<false><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
+                                                                       kept_stride, n_kept, sel_staged_cap(dm));
   ++*launches;
   return cudaGetLastError();
 }
