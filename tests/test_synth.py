@@ -61,3 +61,14 @@ def test_trace_has_spikes_drift_and_band_a_jumps():
     assert 3.0 < g[1] / g[0] < 5.5
     if not sp[t_spike + 1]:
         assert 0.6 < g[2] / g[0] < 1.6
+
+
+def test_pyramid_budgets_recipe():
+    from synth import workloads as W
+    for k_mean, L in ((8192, 32), (4096, 32), (512, 32), (640, 4)):
+        b = W.pyramid_budgets(k_mean, L)
+        assert len(b) == L and all(x % 16 == 0 for x in b)
+        assert all(x >= y for x, y in zip(b, b[1:]))                 # larger budgets for lower layers
+        assert abs(sum(b) / L - k_mean) <= 8                          # the mean stays K (rounding to 16)
+        assert b[0] == round(1.5 * k_mean / 16) * 16 and b[-1] == round(0.5 * k_mean / 16) * 16
+    assert W.pyramid_budgets(100, 1) == (96,)
