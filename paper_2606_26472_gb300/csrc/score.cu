@@ -736,6 +736,10 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
       st.pos[slot] = pos;
       if (dm.kinds & EPIKV_SCORE_BANDZ) st.score[0][slot] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
       if (dm.kinds & EPIKV_SCORE_HSVAR) st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
+      if (dm.layer_budgets) {  // the new token is in every layer
+        st.lmask[slot] = dm.L == 64 ? ~0ull : (1ull << dm.L) - 1ull;
+        for (int l = 0; l < dm.L; ++l) st.n_layer[seq * dm.L + l] += 1;
+      }
       st.n_cache[seq] = nc0 + 1;
       st.n_seen[seq] = pos + 1;
       st.hp_parity[seq] = par ^ 1;

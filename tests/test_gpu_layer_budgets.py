@@ -13,36 +13,11 @@ from paper_2606_26472_gb300 import epikv as E
 from synth import gen, workloads as W
 from synth.device import as_u16
 
-from .harness import OracleTrace, Session, assert_scores_close
+from .harness import LayerReplay, OracleTrace, Session, assert_scores_close
 
 pytestmark = pytest.mark.gpu
 
 BANDZ, LAGKV = E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV
-
-
-class LayerReplay:
-    """The oracle's per-layer caches of one sequence, replayed on the GPU's
-    frozen scores with the same schedule."""
-
-    def __init__(self, n_layers, budgets, prefill, trigger):
-        self.caches = [[] for _ in range(n_layers)]
-        self.budgets, self.prefill, self.trigger = list(budgets), prefill, trigger
-        self.score = {}
-
-    def append(self, positions, scores):
-        for p, s in zip(positions, scores):
-            self.score[int(p)] = float(s)
-        for c in self.caches:
-            c.extend(int(p) for p in positions)
-
-    def event(self):
-        n = max(len(c) for c in self.caches)
-        if not (n > self.trigger and n > min(self.budgets)):
-            return False
-        R = O.layer_recency(self.budgets, self.prefill, n)
-        self.caches = [[c[i] for i in O.select_kept_layer([self.score[p] for p in c], K, self.prefill, R)]
-                       for c, K in zip(self.caches, self.budgets)]
-        return True
 
 
 def _check_layer_bytes(sess, b, layer, positions):
@@ -274,5 +249,37 @@ def test_config2_shape_with_pyramid_layer_budgets(gpu_lib):
             pos = np.asarray(replay[b].caches[l])[slots]
             np.testing.assert_array_equal(k[:, l], gen.kv_rows(m, sess.dt.tabs, b, 0, pos, sp)[:, l])
             np.testing.assert_array_equal(v[:, l], gen.kv_rows(m, sess.dt.tabs, b, 1, pos, sp)[:, l])
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
+def test_layer_budgets_one_token_per_call(gpu_lib):
+    """Decode steps of the band kinds take the fused g + z kernel, which must
+    also advance every layer's length and mark the new slot in every layer."""
+    model = W.small_model(67)
+    L = model.num_layers
+    kinds = BANDZ | E.EPIKV_SCORE_HSVAR
+    budgets = [[60, 40, 50, 30], [45, 45, 20, 70]]
+    triggers = [max(k) + 3 for k in budgets]
+    sess = Session(model, n_seq=2, kinds=kinds, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=80, max_new=1,
+                   prefill=(2, 0), policies=(BANDZ, E.EPIKV_SCORE_HSVAR), layer_budgets=1, layer_tables=True)
+    refs = [OracleTrace(model, sess.dt.tabs, b, 150, kinds) for b in range(2)]
+    replay = [LayerReplay(L, budgets[b], sess.prefill[b], triggers[b]) for b in range(2)]
+    for step in range(150):
+        sess.score_update([(0, 1), (1, 1)])
+        for b in range(2):
+            pos, sc = sess.read(b, sess.policies[b])
+            refs[b].check(sess.policies[b], pos[-1:], sc[-1:], f"seq {b} step {step}")
+            replay[b].append(pos[-1:], sc[-1:])
+        sess.select([0, 1], budgets, triggers)
+        sess.compact([0, 1])
+        for b in range(2):
+            replay[b].event()
+            if step % 10 == 9 or step == 149:
+                for l in range(L):
+                    assert list(sess.read_layer(b, l)) == replay[b].caches[l], f"step {step} seq {b} layer {l}"
+    for b in range(2):
+        for l in range(L):
+            _check_layer_bytes(sess, b, l, replay[b].caches[l])
     assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()

@@ -9,7 +9,7 @@ from paper_2606_26472_gb300 import epikv as E
 from synth import gen, workloads as W
 from synth.device import DeviceTrace, as_u16
 
-from .harness import ALL_KINDS, OracleTrace, Session, assert_scores_close, check_compaction, check_selection
+from .harness import ALL_KINDS, OracleTrace, Session, check_compaction, check_selection
 
 pytestmark = pytest.mark.gpu
 
@@ -97,7 +97,7 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
                     pos, sc = sess.read(b, kind)
                     new = slice(before[b], before[b] + n)
                     np.testing.assert_array_equal(pos[new], np.arange(sess.n_seen[b] - n, sess.n_seen[b]))
-                    assert_scores_close(sc[new], refs[b].scores[kind][pos[new]], f"{name} seq {b} kind {kind}")
+                    refs[b].check(kind, pos[new], sc[new], f"{name} seq {b} kind {kind}")
                     if kind == policies[b]:
                         pre[b] = (pos, sc)
         seqs = [b for b, _ in entries]
@@ -106,8 +106,9 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
         for b, kl in kept.items():
             events += 1
             pos, sc = pre[b]
+            cond = refs[b].cond.get(policies[b])
             check_selection(kl, pos, sc, refs[b].scores[policies[b]][pos], budgets[b], prefill[b], 128,
-                            select_chunk)
+                            select_chunk, None if cond is None else cond[pos])
             pos_after, _ = sess.read(b, policies[b])
             np.testing.assert_array_equal(pos_after, pos[kl])
             check_compaction(sess, b, pos_after)
