@@ -1,10 +1,13 @@
 """Seeded randomised decodes through the C ABI, each drawing its own model
 shape (layers, heads, head size, hidden size, band layers), layout and block
 size, score kinds and selection policies, windows, lag, recency cap,
-prefill, budgets, trigger, new-token pattern, chunk-level selection and
-per-layer budgets (with per-layer block tables), checked against the fp64
-oracle: scores within tolerance, kept lists (or per-layer caches) equal to
-the oracle's on the GPU's own scores, compacted rows equal to the generator's."""
+prefill, budgets, trigger, new-token pattern, skipped sequences, batch
+order, skipped selections, chunk-level selection and per-layer budgets (with
+per-layer block tables), checked against the fp64 oracle: scores within
+tolerance, kept lists (or per-layer caches) equal to the oracle's on the
+GPU's own scores, compacted rows equal to the generator's.  Some trials also
+drive a second context through epikv_step in lockstep and compare the two
+bit for bit."""
 import numpy as np
 import pytest
 
@@ -43,6 +46,10 @@ def _draw(seed):
         lengths=[int(rng.integers(60, 200)) for _ in range(n_seq)],
     )
     p["layer_tables"] = p["layer_budgets"] and p["layout"] == E.EPIKV_LAYOUT_PAGED and bool(rng.integers(0, 2))
+    p["use_step"] = bool(rng.integers(0, 3) == 0)
+    p["select_prob"] = 1.0 if p["use_step"] else float(rng.choice([1.0, 0.6]))
+    p["skip_prob"] = float(rng.choice([0.0, 0.25]))
+    p["shuffle"] = bool(rng.integers(0, 2))
     p["select_chunk"] = 1 if p["layer_budgets"] else int(rng.choice([1, 1, 2, 5]))
     if p["layer_budgets"]:
         p["budgets"] = [[int(x) for x in rng.integers(8, 80, size=L)] for _ in range(n_seq)]
@@ -57,14 +64,20 @@ def test_random_decode_against_the_oracle(gpu_lib, seed):
     m, n_seq, kinds = p["model"], p["n_seq"], p["kinds"]
     kmax = [max(k) if p["layer_budgets"] else k for k in p["budgets"]]
     max_new = max(p["chunks"])
-    T_cap = max(max(kmax) + p["slack"], max(p["prefill"])) + max_new + 1
+    T_cap = max(max(kmax) + p["slack"], max(p["prefill"])) + 4 * max_new + 1   # room for skipped selections
     sess = Session(m, n_seq=n_seq, kinds=kinds, layout=p["layout"], max_tokens=T_cap, max_new=max_new,
                    prefill=p["prefill"], policies=p["policies"], z_window=p["z_window"], lag=p["lag"],
                    lag_window=p["lag_window"], recency_cap=p["cap"], block_size=p["block_size"],
                    select_chunk=p["select_chunk"], layer_budgets=int(p["layer_budgets"]),
                    layer_tables=p["layer_tables"])
+    twin = Session(m, n_seq=n_seq, kinds=kinds, layout=p["layout"], max_tokens=T_cap, max_new=max_new,
+                   prefill=p["prefill"], policies=p["policies"], z_window=p["z_window"], lag=p["lag"],
+                   lag_window=p["lag_window"], recency_cap=p["cap"], block_size=p["block_size"],
+                   select_chunk=p["select_chunk"], layer_budgets=int(p["layer_budgets"]),
+                   layer_tables=p["layer_tables"]) if p["use_step"] else None
     refs = [OracleTrace(m, sess.dt.tabs, b, p["lengths"][b], kinds, z_window=p["z_window"], lag=p["lag"],
                         lag_window=p["lag_window"]) for b in range(n_seq)]
+    srng = np.random.default_rng(seed + 1000)
     triggers = [kmax[b] + p["slack"] for b in range(n_seq)]
     replay = [LayerReplay(m.num_layers, p["budgets"][b], p["prefill"][b],
                           triggers[b] if p["use_trigger"] else kmax[b]) for b in range(n_seq)] \
@@ -73,6 +86,11 @@ def test_random_decode_against_the_oracle(gpu_lib, seed):
     while any(sess.n_seen[b] < p["lengths"][b] for b in range(n_seq)):
         entries = [(b, min(p["chunks"][(b + step) % 3], p["lengths"][b] - sess.n_seen[b])) for b in range(n_seq)
                    if sess.n_seen[b] < p["lengths"][b]]
+        if len(entries) > 1 and p["skip_prob"] > 0:   # some sequences bring nothing this step
+            kept_entries = [e for e in entries if srng.random() >= p["skip_prob"]]
+            entries = kept_entries or entries[:1]
+        if p["shuffle"]:
+            entries = [entries[i] for i in srng.permutation(len(entries))]
         step += 1
         before = {b: sess.n_cache[b] for b, _ in entries}
         sess.score_update(entries)
@@ -91,8 +109,24 @@ def test_random_decode_against_the_oracle(gpu_lib, seed):
                         replay[b].append(pos[new], sc[new])
         seqs = [b for b, _ in entries]
         trig = [triggers[b] for b in seqs] if p["use_trigger"] else None
+        if twin is not None:   # the same step through epikv_step (no trigger = the budget, K_max per layer)
+            twin.step(entries, [p["budgets"][b] for b in seqs], trig or [kmax[b] for b in seqs])
+        full = any(sess.n_cache[b] + 2 * max_new > T_cap for b in seqs)   # must evict before it overflows
+        if not full and srng.random() >= p["select_prob"]:
+            continue
         kept = sess.select(seqs, [p["budgets"][b] for b in seqs], trig)
         sess.compact(seqs)
+        if twin is not None:
+            for b in seqs:
+                assert twin.n_cache[b] == sess.n_cache[b], (seed, step, b)
+                if p["layer_budgets"]:
+                    assert twin.n_layer[b] == sess.n_layer[b], (seed, step, b)
+                for kind in ALL_KINDS:
+                    if kinds & kind:
+                        pa, sa = sess.read(b, kind)
+                        pb, sb = twin.read(b, kind)
+                        np.testing.assert_array_equal(pa, pb)
+                        np.testing.assert_array_equal(sa.view(np.uint32), sb.view(np.uint32))
         for b in seqs:
             if replay:
                 replay[b].event(p["cap"])
@@ -115,5 +149,18 @@ def test_random_decode_against_the_oracle(gpu_lib, seed):
                 sp = gen.spike_flags(m, b, int(pos.max()) + 1)
                 np.testing.assert_array_equal(k, gen.kv_rows(m, sess.dt.tabs, b, 0, pos, sp)[:, l])
                 np.testing.assert_array_equal(v, gen.kv_rows(m, sess.dt.tabs, b, 1, pos, sp)[:, l])
+    if twin is not None:
+        for b in range(n_seq):
+            n = twin.n_cache[b]
+            if p["layer_budgets"]:
+                for l in range(m.num_layers):
+                    nl = twin.n_layer[b][l]
+                    np.testing.assert_array_equal(np.stack(twin.layer_rows_u16(b, l, np.arange(nl))),
+                                                  np.stack(sess.layer_rows_u16(b, l, np.arange(nl))))
+            else:
+                np.testing.assert_array_equal(np.stack(twin.cache_rows_u16(b, np.arange(n))),
+                                              np.stack(sess.cache_rows_u16(b, np.arange(n))))
+        assert twin.error() == (E.EPIKV_OK, 0)
+        twin.close()
     assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()
