@@ -471,7 +471,7 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src,
                      "traffic": traffic, "algorithmic_bytes_per_launch": compact_bytes / args.steps},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": 5 * args.steps,   # Lag-KV partial, finalize, select, compaction, eviction consumed
         "clocks": clk,
         "e2e": e2e,
     }
@@ -577,7 +577,7 @@ def run_bandz2k(args):
             "roofline": {"bound": "hbm", "kernel": "score phase (bandz_g_kernel + score_finalize_kernel)",
                          "achieved": g, "peak": peak, "unit": "GB/s", "frac": g / peak, "peak_source": peak_src,
                          "traffic": None, "algorithmic_bytes_per_launch": score_bytes},
-            "gpu_launches": 5 * args.steps}
+            "gpu_launches": 6 * args.steps}   # reset, g, finalize, select, compaction, eviction consumed
     print(json.dumps(line), flush=True)
 
 
@@ -816,7 +816,7 @@ def run_layers32k(args):
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src, "traffic": None,
                      "algorithmic_bytes_per_launch": compact_bytes / args.steps},
-        "gpu_launches": 5 * args.steps,   # Lag-KV partial, finalize, layer keep, layer union, compaction
+        "gpu_launches": 6 * args.steps,   # Lag-KV partial, finalize, layer keep, layer union, compaction, consumed
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

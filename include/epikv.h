@@ -229,7 +229,10 @@ epikv_status epikv_select(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_id
 /* Move every layer's K and V rows of the entries that evicted in the
  * preceding epikv_select to their kept slots, in order, in place (App. H).
  * Rows before the first evicted slot are not touched.  d_kept has the layout
- * epikv_select wrote (per layer with cfg.layer_budgets = 1). */
+ * epikv_select wrote (per layer with cfg.layer_budgets = 1).  An eviction is
+ * applied once: calling epikv_compact again, or with no eviction selected
+ * since the last score update, moves nothing; a score update that finds an
+ * eviction selected but not yet compacted reports EPIKV_DEV_KEPT. */
 epikv_status epikv_compact(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
                            const int32_t* d_kept, int32_t kept_stride, const epikv_kv_view* kv,
                            cudaStream_t stream);

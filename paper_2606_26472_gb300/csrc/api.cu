@@ -133,8 +133,8 @@ size_t carve(const Dims& d, DevState* st, char* base) {
     st->lmask_new = (unsigned long long*)take(S * T * 8);
     st->lkeep = (uint32_t*)take(S * d.L * ((T + 31) / 32) * 4);
     st->mkept = (int32_t*)take(S * T * 4);
-    st->work = (uint32_t*)take(2 * 4);
   }
+  st->work = (uint32_t*)take(2 * 4);
   return align_up(off, 256);
 }
 

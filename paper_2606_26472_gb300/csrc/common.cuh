@@ -61,7 +61,7 @@ struct DevState {
   unsigned long long* lmask_new;  // [S][T] the select kernel's new masks (scratch)
   uint32_t* lkeep;         // [S][L][ceil(T/32)] bit: layer l keeps the union slot (scratch)
   int32_t* mkept;          // [S][T] the select kernel's kept slots of the largest layer (scratch)
-  uint32_t* work;          // [2] the per-layer compaction's next unit and finished CTAs (0 between launches)
+  uint32_t* work;          // [2] the compaction's next unit (per-layer budgets) and finished CTAs (0 between launches)
 };
 
 struct Dims {

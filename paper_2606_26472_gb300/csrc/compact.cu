@@ -20,6 +20,10 @@
 // the CTAs take units from a shared counter instead of a fixed stride, in
 // layer-major order: with budgets that fall with depth, larger streams come
 // first and the greedy assignment ends nearly level.
+//
+// A selection's eviction is compacted once: compact_consumed_kernel, launched
+// after the copy, sets each sequence's first moved slot to its length, so
+// another compaction before the next selection moves nothing.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -274,6 +278,17 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   }
 }
 
+// The batch entries' evictions have been applied: nothing is left pending.
+__global__ void compact_consumed_kernel(DevState st, Dims dm, const int32_t* __restrict__ seq_ids, int n_seq) {
+  for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < n_seq; b += gridDim.x * blockDim.x) {
+    const int seq = seq_ids[b];
+    if (seq < 0 || seq >= dm.S) continue;
+    st.first_changed[seq] = st.n_cache[seq];
+    if (dm.layer_budgets)
+      for (int l = 0; l < dm.L; ++l) st.lfirst[seq * dm.L + l] = st.n_layer[seq * dm.L + l];
+  }
+}
+
 static int g_ctas_per_sm = 0;
 
 static size_t compact_smem(int n_seq) {
@@ -306,6 +321,10 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
     compact_kernel<true><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
   else
     compact_kernel<false><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  ++*launches;
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  compact_consumed_kernel<<<(n_seq + 255) / 256, 256, 0, stream>>>(st, dm, seq_ids, n_seq);
   ++*launches;
   return cudaGetLastError();
 }

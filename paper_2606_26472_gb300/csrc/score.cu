@@ -594,10 +594,17 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
     if (done == gridDim.x - 1) {
       __threadfence();
       if (fits) {
+        // an eviction selected but not compacted before this update breaks the
+        // call order; nothing is left pending for a later compaction either way
+        if (st.first_changed[seq] < nc0) set_error(st.err, EPIKV_DEV_KEPT);
+        st.first_changed[seq] = nc0 + n_new;
         st.n_cache[seq] = nc0 + n_new;
         st.n_seen[seq] = p0 + n_new;
         if (dm.layer_budgets)
-          for (int l = 0; l < dm.L; ++l) st.n_layer[seq * dm.L + l] += n_new;
+          for (int l = 0; l < dm.L; ++l) {
+            st.n_layer[seq * dm.L + l] += n_new;
+            st.lfirst[seq * dm.L + l] = st.n_layer[seq * dm.L + l];
+          }
         if ((dm.kinds & kBandKinds) && n_new > 0) st.hp_parity[seq] ^= 1;
         atomicAdd(&st.stats[0], (unsigned long long)n_new);
       }
@@ -738,8 +745,13 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
       if (dm.kinds & EPIKV_SCORE_HSVAR) st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
       if (dm.layer_budgets) {  // the new token is in every layer
         st.lmask[slot] = dm.L == 64 ? ~0ull : (1ull << dm.L) - 1ull;
-        for (int l = 0; l < dm.L; ++l) st.n_layer[seq * dm.L + l] += 1;
+        for (int l = 0; l < dm.L; ++l) {
+          st.n_layer[seq * dm.L + l] += 1;
+          st.lfirst[seq * dm.L + l] = st.n_layer[seq * dm.L + l];
+        }
       }
+      if (st.first_changed[seq] < nc0) set_error(st.err, EPIKV_DEV_KEPT);  // as in score_finalize_kernel
+      st.first_changed[seq] = nc0 + 1;
       st.n_cache[seq] = nc0 + 1;
       st.n_seen[seq] = pos + 1;
       st.hp_parity[seq] = par ^ 1;

@@ -265,8 +265,9 @@ class Session:
         return out
 
     def compact(self, seqs):
-        seq_ids = self._sel[0]
+        seq_ids = torch.tensor(seqs, dtype=torch.int32, device=self.ws.device)
         E.epikv_compact(self.ctx, len(seqs), seq_ids, self.kept, self.kept.shape[-1], self.kv)
+        self._cmp = seq_ids
 
     def read_layer(self, b, layer):
         pos, n = E.epikv_read_layer_slots(self.ctx, b, layer, self.cache.T)

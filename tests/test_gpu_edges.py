@@ -7,7 +7,7 @@ import torch
 
 from oracle import epikv_oracle as O
 from paper_2606_26472_gb300 import epikv as E
-from synth import workloads as W
+from synth import gen, workloads as W
 
 from .harness import OracleTrace, Session, assert_scores_close, check_compaction
 
@@ -91,4 +91,39 @@ def test_nan_scores_rank_lowest(gpu_lib):
     kept = sess.select([0], [K])[0]
     assert list(kept) == O.select_kept(sc.astype(np.float64), K, 0, 128)
     assert not set(range(50, 115)) & set(kept[:-17])     # NaN candidates lose to every number
+    sess.close()
+
+
+@pytest.mark.parametrize("layer_budgets", [0, 1], ids=["token", "per_layer"])
+def test_a_compaction_is_applied_once(gpu_lib, layer_budgets):
+    """A selection's eviction is compacted once: a second epikv_compact (or
+    one after a score update with no selection) leaves the cache alone."""
+    model = W.small_model(45)
+    sess = Session(model, n_seq=2, kinds=KINDS, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=120, max_new=100,
+                   prefill=(0, 3), policies=(1, 2), layer_budgets=layer_budgets)
+    budgets = [[40, 30, 50, 20], [60, 60, 25, 35]] if layer_budgets else [40, 60]
+
+    def snapshot():
+        return [np.stack(sess.cache_rows_u16(b, np.arange(sess.n_cache[b]))) for b in range(2)]
+
+    sess.score_update([(0, 100), (1, 90)])
+    sess.compact([0, 1])                     # nothing selected yet: nothing moves
+    sess.select([0, 1], budgets)
+    first = snapshot()
+    sess.compact([0, 1])
+    after = snapshot()
+    sess.compact([0, 1])                     # the same eviction again: a no-op
+    again = snapshot()
+    for b in range(2):
+        np.testing.assert_array_equal(after[b], again[b])
+        assert not np.array_equal(first[b], after[b])    # the first compaction did move rows
+        if layer_budgets:
+            for l in range(model.num_layers):
+                pos = sess.read_layer(b, l)
+                k, v = sess.layer_rows_u16(b, l, np.arange(len(pos)))
+                sp = gen.spike_flags(model, b, int(pos.max()) + 1)
+                np.testing.assert_array_equal(k, gen.kv_rows(model, sess.dt.tabs, b, 0, pos, sp)[:, l])
+        else:
+            check_compaction(sess, b, sess.read(b, 1)[0])
+    assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()
