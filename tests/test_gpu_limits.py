@@ -1,0 +1,85 @@
+"""The path at the limits of its configuration: an 8192-wide hidden state (four
+16-byte vectors per thread in the g kernels, multi-token and one-token
+calls), 32 band layers with a 1,024-token z window and a 1,024-token K/V
+window (the finalize kernel's largest shared-memory staging), and a batch of
+300 sequences in one call.  Scores against the fp64 oracle, kept lists
+against the oracle's selection on the GPU's own scores, compacted rows
+against the generator."""
+import numpy as np
+import pytest
+
+from paper_2606_26472_gb300 import epikv as E
+from synth import gen
+
+from .harness import OracleTrace, Session, check_compaction, check_selection
+
+pytestmark = pytest.mark.gpu
+
+BANDZ, LAGKV, HSVAR = E.EPIKV_SCORE_BANDZ, E.EPIKV_SCORE_LAGKV, E.EPIKV_SCORE_HSVAR
+
+
+@pytest.mark.parametrize("chunk", [1, 37], ids=["one_token_calls", "multi_token_calls"])
+def test_widest_hidden_state(gpu_lib, chunk):
+    model = gen.TraceModel(0xE91C0201, num_layers=3, hidden=8192, num_kv_heads=1, head_dim=8,
+                           band_a=(0,), band_b=(1, 2))
+    T = 150
+    kinds = BANDZ | HSVAR
+    sess = Session(model, n_seq=2, kinds=kinds, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=T, max_new=chunk,
+                   prefill=(0, 0), policies=(BANDZ, HSVAR))
+    refs = [OracleTrace(model, sess.dt.tabs, b, T, kinds) for b in range(2)]
+    while sess.n_seen[0] < T:
+        n = min(chunk, T - sess.n_seen[0])
+        sess.score_update([(0, n), (1, n)])
+    for b in range(2):
+        for kind in (BANDZ, HSVAR):
+            pos, sc = sess.read(b, kind)
+            refs[b].check(kind, pos, sc, f"D=8192 seq {b} kind {kind}")
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
+def test_largest_windows_and_band_count(gpu_lib):
+    model = gen.TraceModel(0xE91C0202, num_layers=32, hidden=64, num_kv_heads=1, head_dim=8,
+                           band_a=tuple(range(16)), band_b=tuple(range(16, 32)))
+    T, K = 1300, 700
+    kinds = BANDZ | HSVAR | LAGKV
+    sess = Session(model, n_seq=1, kinds=kinds, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=T, max_new=400,
+                   prefill=(3,), policies=(BANDZ,), z_window=1024, lag_window=1024)
+    ref = OracleTrace(model, sess.dt.tabs, 0, T, kinds, z_window=1024, lag_window=1024)
+    while sess.n_seen[0] < T:
+        sess.score_update([(0, min(400, T - sess.n_seen[0]))])
+    pos, sc = sess.read(0, BANDZ)
+    for kind in (BANDZ, HSVAR, LAGKV):
+        p_, s_ = sess.read(0, kind)
+        ref.check(kind, p_, s_, f"32 bands, windows 1024, kind {kind}")
+    kept = sess.select([0], [K])[0]
+    sess.compact([0])
+    check_selection(kept, pos, sc, ref.scores[BANDZ][pos], K, 3, 128, 1, ref.cond[BANDZ][pos])
+    check_compaction(sess, 0, sess.read(0, BANDZ)[0])
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
+def test_three_hundred_sequences_in_one_call(gpu_lib):
+    model = gen.TraceModel(0xE91C0203, num_layers=2, hidden=64, num_kv_heads=1, head_dim=16,
+                           band_a=(0,), band_b=(1,))
+    S, T, K = 300, 48, 20
+    kinds = BANDZ | LAGKV
+    policies = [BANDZ if b % 2 else LAGKV for b in range(S)]
+    sess = Session(model, n_seq=S, kinds=kinds, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=T, max_new=T,
+                   prefill=[b % 3 for b in range(S)], policies=policies, block_size=4)
+    sess.score_update([(b, T - (b % 7)) for b in range(S)])
+    pre = {b: sess.read(b, policies[b]) for b in range(S)}
+    kept = sess.select(list(range(S)), [K + (b % 5) for b in range(S)])
+    sess.compact(list(range(S)))
+    assert len(kept) == S
+    rng = np.random.default_rng(3)
+    for b in sorted(rng.choice(S, size=40, replace=False)):
+        pos, sc = pre[b]
+        ref = OracleTrace(model, sess.dt.tabs, b, T - (b % 7), kinds)
+        ref.check(policies[b], pos, sc, f"seq {b}")
+        check_selection(kept[b], pos, sc, ref.scores[policies[b]][pos], K + (b % 5), b % 3, 128, 1,
+                        ref.cond[BANDZ][pos] if policies[b] == BANDZ else None)
+        check_compaction(sess, b, sess.read(b, policies[b])[0])
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
