@@ -61,7 +61,7 @@ def parse():
     p.add_argument("--chunk", type=int, default=128)
     # the band-z kernels' workload: the 2,048-token single-sequence case, one
     # fresh sequence per step (reported for the per-kernel rooflines)
-    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken", "layers32k"])
+    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken", "layers32k", "bandz8k", "ragged64"])
     # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
     # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
     p.add_argument("--kinds", type=int, default=2)
@@ -122,6 +122,15 @@ class Clocks:
     def __init__(self, gpu_id):
         self.gpu_id = gpu_id   # the device's UUID ("GPU-...") so no other GPU is sampled
         self.proc = None
+
+    @staticmethod
+    def device_id(dev, local_rank):
+        """nvidia-smi's --id for torch device `dev`: its UUID, else the local rank."""
+        try:
+            uuid = str(torch.cuda.get_device_properties(dev).uuid)
+            return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+        except Exception:
+            return str(local_rank)
 
     def start(self):
         self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
@@ -333,11 +342,7 @@ def run_ours(args):
     phase = [new_events() for _ in range(args.steps)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    try:
-        uuid = str(torch.cuda.get_device_properties(dev).uuid)
-        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
-    except Exception:
-        gpu_id = str(local_rank)
+    gpu_id = Clocks.device_id(dev, local_rank)
     clocks = Clocks(gpu_id)
     clocks.start()
     if world > 1:
@@ -761,11 +766,7 @@ def run_layers32k(args):
     phase = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_steps)]
     for e in (x for p in phase for x in p):
         e.record(stream)   # materialise the handles
-    try:
-        uuid = str(torch.cuda.get_device_properties(dev).uuid)
-        gpu_id = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
-    except Exception:
-        gpu_id = str(local_rank)
+    gpu_id = Clocks.device_id(dev, local_rank)
     clocks = None
     stats0 = None
     for st in range(n_steps):
@@ -822,6 +823,213 @@ def run_layers32k(args):
     print(json.dumps(line), flush=True)
 
 
+def run_window(args):
+    """Steady-state decode windows of two more workloads, timed per
+    epikv_step call with CUDA events on the stream; the generator kernels
+    that append each call's new rows (the model's side of the loop) run
+    between the events:
+    * bandz8k: 8 x 8,192-token band-z traces, contiguous K/V, K = 4,096;
+      64 new tokens per sequence per call, every call evicts back to K;
+    * ragged64: 64 sequences with budgets from {2048, 4096, 8192}, paged
+      16-token blocks, both scores, one new token per sequence per call; a
+      sequence evicts when its cache exceeds K + 64.  The sequences start at
+      staggered lengths K + (29 b mod 65), so one of them evicts at nearly
+      every call.
+    One bench step = the calls in which every sequence evicts once (1 and
+    65).  Every call has the same arguments, so one captured CUDA graph of
+    the call is replayed; the eager rate (with the per-phase breakdown) is
+    reported beside it."""
+    import torch
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    from paper_2606_26472_gb300.cache import KVCache
+    from synth import gen, workloads as W
+    from synth.device import DeviceBatchTrace
+
+    rank, local_rank, world = dist_env()
+    assert world == 1, "the decode-window workloads are single-GPU measurements"
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+    ragged = args.workload == "ragged64"
+    wl = W.config(5 if ragged else 2)
+    m = wl.model
+    L, H, d, nb = m.num_layers, m.num_kv_heads, m.head_dim, len(m.band_layers)
+    Bn, C = wl.n_seq, wl.chunk
+    budgets = np.array(wl.budgets, dtype=np.int64)
+    slack = wl.trigger_slack[0]
+    assert all(s == slack for s in wl.trigger_slack)
+    cycle = slack + 1                   # new tokens of a sequence between two of its evictions
+    calls = cycle // C                  # calls per bench step
+    assert calls * C == cycle
+    phase0 = (np.arange(Bn) * 29) % cycle if C == 1 else np.zeros(Bn, np.int64)
+    n0 = budgets + phase0
+    T_cap = int(budgets.max()) + cycle
+    n_calls = 2 * (args.warmup + args.steps) * calls      # eager run, then graph run
+    max_pos = int(n0.max()) + n_calls * C + 1
+    paged = wl.layout == W.PAGED
+    if paged:
+        mb = (T_cap + wl.block_size - 1) // wl.block_size
+        bt = gen.block_permutation(m.seed, Bn * mb).reshape(Bn, mb)
+        cache = KVCache(E.EPIKV_LAYOUT_PAGED, L, H, d, max_seqs=Bn, max_tokens=T_cap, block_size=wl.block_size,
+                        block_table=bt, device=dev)
+    else:
+        cache = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, L, H, d, max_seqs=Bn, max_tokens=T_cap, device=dev)
+    kv = cache.view()
+    setup_chunk = 256
+    cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T_cap, max_new_tokens=max(setup_chunk, C), num_layers=L,
+                        num_kv_heads=H, head_dim=d, hidden=m.hidden, n_band_a=len(m.band_a),
+                        n_band_b=len(m.band_b), z_window=wl.z_window, lag=wl.lag, lag_window=wl.lag_window,
+                        recency_cap=wl.recency_cap, score_kinds=wl.kinds)
+    ws = torch.empty(E.epikv_workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws.numel())
+    for b in range(Bn):
+        E.epikv_seq_reset(ctx, b, 0, wl.policies[b])
+    dt = DeviceBatchTrace(m, Bn, max_pos, dev)
+
+    # every sequence's first n0 tokens, scored in chunks (no eviction yet)
+    hs = torch.empty((nb, setup_chunk, m.hidden), dtype=torch.bfloat16, device=dev)
+    hv_s = E.hidden_view([hs[i] for i in range(nb)], m.hidden)
+    cu_s = {}
+    for b in range(Bn):
+        ids = torch.tensor([b], dtype=torch.int32, device=dev)
+        for p0 in range(0, int(n0[b]), setup_chunk):
+            c = min(setup_chunk, int(n0[b]) - p0)
+            if c not in cu_s:
+                cu_s[c] = torch.tensor([0, c], dtype=torch.int32, device=dev)
+            for i, layer in enumerate(m.band_layers):
+                dt.hidden(b, layer, p0, c, hs[i], m.hidden)
+            dt.kv(b, p0, c, p0, cache.k, cache.v, **cache.synth_kwargs())
+            E.epikv_score_update(ctx, 1, ids, cu_s[c], c, hv_s, kv)
+
+    # each call's rows: (sequence, position, slot), simulated on the host
+    n_cache = n0.copy()
+    pos_tab = np.empty((n_calls, Bn * C), np.int32)
+    slot_tab = np.empty((n_calls, Bn * C), np.int32)
+    evict_tab = np.zeros(n_calls, np.int64)
+    r = np.arange(C)
+    for j in range(n_calls):
+        pos_tab[j] = (n0[:, None] + j * C + r[None, :]).reshape(-1)
+        slot_tab[j] = (n_cache[:, None] + r[None, :]).reshape(-1)
+        n_cache += C
+        ev = n_cache > budgets + slack
+        evict_tab[j] = int(ev.sum())
+        n_cache[ev] = budgets[ev]
+    seq_rows = torch.from_numpy(np.repeat(np.arange(Bn, dtype=np.int32), C)).to(dev)
+    pos_dev = torch.from_numpy(pos_tab).to(dev)
+    slot_dev = torch.from_numpy(slot_tab).to(dev)
+    hid = torch.empty((nb, Bn * C, m.hidden), dtype=torch.bfloat16, device=dev)
+    hv = E.hidden_view([hid[i] for i in range(nb)], m.hidden)
+    seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
+    cu = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * C).contiguous()
+    bud = torch.from_numpy(budgets.astype(np.int32)).to(dev)
+    trig = (bud + slack).contiguous()
+    n_out = torch.empty(Bn, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code} during set-up"
+
+    def append(j):   # call j's new rows: hidden rows of the band layers, K/V into their slots
+        for i, layer in enumerate(m.band_layers):
+            dt.hidden_batch(layer, seq_rows, pos_dev[j], hid[i], m.hidden)
+        dt.kv_batch(seq_rows, pos_dev[j], slot_dev[j], cache.k, cache.v, **cache.synth_kwargs())
+
+    def call():
+        E.epikv_step(ctx, Bn, seq_ids, cu, C, bud, trig, hv, kv, n_out)
+
+    j = 0
+
+    def window(n_steps, run, timed, phases=False):
+        nonlocal j
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(n_steps * calls)] if timed else []
+        ph = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_steps * calls)] \
+            if phases else []
+        for p in ph:
+            for e in p:
+                e.record(stream)   # materialise the handles
+        for k in range(n_steps * calls):
+            append(j)
+            if ph:
+                E.epikv_set_phase_events(ctx, ph[k])
+            if ev:
+                # ~0.1 ms of device spin ahead of the start event: the whole
+                # call is queued before the device reaches it, so no host
+                # submission gap falls between the events
+                torch.cuda._sleep(200000)
+                ev[k][0].record(stream)
+            run()
+            if ev:
+                ev[k][1].record(stream)
+            j += 1
+        torch.cuda.synchronize()
+        E.epikv_set_phase_events(ctx, None)
+        ms = sum(a.elapsed_time(b_) for a, b_ in ev)
+        per_phase = [sum(p[q].elapsed_time(p[q + 1]) for p in ph) for q in range(3)] if ph else None
+        return ms, per_phase
+
+    gpu_id = Clocks.device_id(dev, local_rank)
+    window(args.warmup, call, False)
+    s0 = E.epikv_get_stats(ctx)
+    j0 = j
+    ms_eager, (t_score, t_select, t_compact) = window(args.steps, call, True, phases=True)
+    s1 = E.epikv_get_stats(ctx)
+    assert s1["evictions"] - s0["evictions"] == int(evict_tab[j0:j].sum())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        call()
+    window(args.warmup, g.replay, False)
+    clocks = Clocks(gpu_id)
+    clocks.start()
+    s2 = E.epikv_get_stats(ctx)
+    j2 = j
+    ms_graph, _ = window(args.steps, g.replay, True)
+    clk = clocks.stop()
+    s3 = E.epikv_get_stats(ctx)
+    assert j == n_calls
+    assert s3["evictions"] - s2["evictions"] == int(evict_tab[j2:j].sum())
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    for b in range(Bn):   # the device's cache lengths follow the host's simulation
+        _, _, n = E.epikv_read_slots(ctx, b, wl.policies[b], 1)
+        assert n == n_cache[b], (b, n, int(n_cache[b]))
+
+    tokens = args.steps * calls * Bn * C
+    assert s3["tokens_scored"] - s2["tokens_scored"] == tokens
+    row_bytes = L * 2 * H * d * 2
+    rows = s1["rows_moved"] - s0["rows_moved"]
+    compact_bytes = 2 * rows * row_bytes
+    n_launch = calls * args.steps
+    peak, peak_src = measured_hbm_peak()
+    ach = compact_bytes / (t_compact / 1e3) / 1e9
+    workload = ("ragged64_4k32k_both_paged16_steady" if ragged else "batch8_8k_bandz_contiguous_K4096_every64")
+    line = {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_graph / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": workload, "sequences": Bn, "budgets": sorted(set(wl.budgets)),
+                       "new_tokens_per_call": C, "calls_per_step": calls,
+                       "evict_when": f"n_cache > K + {slack}", "layout": "paged16_shuffled" if paged else "contiguous",
+                       "score_kinds": wl.kinds, "timing": "CUDA events around each epikv_step call, queued behind a device spin",
+                       "l2": "K/V caches %.1f GiB, larger than L2" % (cache.k.numel() * 4 / 2 ** 30)},
+            "eager_value": tokens / (ms_eager / 1e3),
+            "us_per_call": {"graph": 1e3 * ms_graph / n_launch, "eager": 1e3 * ms_eager / n_launch},
+            "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
+                                    "compact": t_compact / args.steps},
+            "evictions_per_step": (s1["evictions"] - s0["evictions"]) / args.steps,
+            "compaction_gbs": ach,
+            "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
+                         "frac": ach / peak, "peak_source": peak_src, "traffic": None,
+                         "algorithmic_bytes_per_launch": compact_bytes / n_launch,
+                         "timing": "eager calls, phase events"},
+            "gpu_launches": (6 if wl.kinds & E.EPIKV_SCORE_LAGKV else 5) * n_launch,
+            "clocks": clk}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -832,6 +1040,8 @@ def main():
         run_pertoken(args)
     elif args.workload == "layers32k":
         run_layers32k(args)
+    elif args.workload in ("bandz8k", "ragged64"):
+        run_window(args)
     else:
         run_ours(args)
 

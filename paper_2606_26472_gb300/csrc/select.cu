@@ -95,6 +95,35 @@ __device__ __forceinline__ int block_min(int v, int* sh) {
   return r;
 }
 
+// Slot j <- slot kept[j] of the sequence's scores (every kind) and positions,
+// for j from fe to n_kept, in place: safe in increasing j because kept[j] >= j
+// and each round reads all its sources before any of its stores.  Every
+// thread of the block calls it.
+__device__ __forceinline__ void compact_metadata(const DevState& st, const Dims& dm, int seq,
+                                                 const int32_t* __restrict__ kept, int fe, int n_kept) {
+  const int tid = threadIdx.x;
+  int32_t* ps = st.pos + (size_t)seq * dm.T;
+  for (int j0 = fe; j0 < n_kept; j0 += kSelThreads) {
+    const int j = j0 + tid;
+    float v[kNumKinds];
+    int32_t p = 0;
+    if (j < n_kept) {
+      const int src = kept[j];
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k) v[k] = st.score[k] ? st.score[k][(size_t)seq * dm.T + src] : 0.f;
+      p = ps[src];
+    }
+    __syncthreads();
+    if (j < n_kept) {
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k)
+        if (st.score[k]) st.score[k][(size_t)seq * dm.T + j] = v[k];
+      ps[j] = p;
+    }
+    __syncthreads();
+  }
+}
+
 struct RadixShared {
   uint32_t hist[256];
   uint32_t prefix, mask, remaining;
@@ -278,26 +307,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   __syncthreads();  // kept list visible to the whole block
 
   // ---- compact slot metadata in place (kept[i] >= i, increasing i)
-  int32_t* ps = st.pos + (size_t)seq * dm.T;
-  for (int j0 = fe; j0 < n_kept; j0 += kSelThreads) {
-    const int j = j0 + tid;
-    float v[kNumKinds];
-    int32_t p = 0;
-    if (j < n_kept) {
-      const int src = out[j];
-#pragma unroll
-      for (int k = 0; k < kNumKinds; ++k) v[k] = st.score[k] ? st.score[k][(size_t)seq * dm.T + src] : 0.f;
-      p = ps[src];
-    }
-    __syncthreads();
-    if (j < n_kept) {
-#pragma unroll
-      for (int k = 0; k < kNumKinds; ++k)
-        if (st.score[k]) st.score[k][(size_t)seq * dm.T + j] = v[k];
-      ps[j] = p;
-    }
-    __syncthreads();
-  }
+  compact_metadata(st, dm, seq, out, fe, n_kept);
   if (tid == 0) {
     st.n_cache[seq] = n_kept;
     st.first_changed[seq] = fe;
@@ -557,26 +567,7 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
   }
   fe = min(block_min(fe, sh_scan), n_union);
   __syncthreads();  // the union's kept list is visible to the whole block
-  int32_t* ps = st.pos + (size_t)seq * dm.T;
-  for (int j0 = fe; j0 < n_union; j0 += kSelThreads) {
-    const int j = j0 + tid;
-    float v[kNumKinds];
-    int32_t p = 0;
-    if (j < n_union) {
-      const int src = mkept[j];
-#pragma unroll
-      for (int k = 0; k < kNumKinds; ++k) v[k] = st.score[k] ? st.score[k][(size_t)seq * dm.T + src] : 0.f;
-      p = ps[src];
-    }
-    __syncthreads();
-    if (j < n_union) {
-#pragma unroll
-      for (int k = 0; k < kNumKinds; ++k)
-        if (st.score[k]) st.score[k][(size_t)seq * dm.T + j] = v[k];
-      ps[j] = p;
-    }
-    __syncthreads();
-  }
+  compact_metadata(st, dm, seq, mkept, fe, n_union);
   // every new mask lands in its slot (the slots before fe did not move)
   for (int j = tid; j < n_union; j += kSelThreads) mk[j] = mn[mkept[j]];
   if (tid == 0) {
