@@ -83,6 +83,7 @@ Dims make_dims(const epikv_config* c) {
   d.lag_window = lg ? c->lag_window : 1;
   d.lag_eps = c->lag_eps;
   // rings hold every position a window of this call can reach (see finalize)
+  d.stash_rows = d.T < kStashRows ? d.T : kStashRows;
   d.G = next_pow2(c->max_new_tokens + (d.z_window > d.lag_window ? d.z_window : d.lag_window));
   return d;
 }
@@ -135,6 +136,7 @@ size_t carve(const Dims& d, DevState* st, char* base) {
     st->mkept = (int32_t*)take(S * T * 4);
   }
   st->work = (uint32_t*)take(2 * 4);
+  st->stash = (char*)take((size_t)kMaxStashCtas * d.stash_rows * d.H * d.d * 2);
   return align_up(off, 256);
 }
 

@@ -62,10 +62,17 @@ struct DevState {
   uint32_t* lkeep;         // [S][L][ceil(T/32)] bit: layer l keeps the union slot (scratch)
   int32_t* mkept;          // [S][T] the select kernel's kept slots of the largest layer (scratch)
   uint32_t* work;          // [2] the compaction's next unit (per-layer budgets) and finished CTAs (0 between launches)
+  char* stash;             // [kMaxStashCtas][stash_rows][H*d] bf16: compaction boundary rows (token budgets)
 };
+
+// The balanced compaction split: at most this many CTAs, each with a stash
+// of at most kStashRows rows (the slots its left neighbour still reads).
+constexpr int kMaxStashCtas = 512;
+constexpr int kStashRows = 128;
 
 struct Dims {
   int S, T, max_new, L, H, d, D, nA, nB, G;
+  int stash_rows;  // min(kStashRows, T): rows of one CTA's compaction stash
   int z_window, lag, lag_window, recency_cap, kinds, select_chunk, layer_budgets;
   float z_eps, lag_eps;
 };

@@ -21,6 +21,16 @@
 // layer-major order: with budgets that fall with depth, larger streams come
 // first and the greedy assignment ends nearly level.
 //
+// Balanced split (token budgets): the moved rows of all evicting streams,
+// laid end to end, are cut into one equal chunk per CTA, so one evicting
+// sequence still covers the whole grid and no CTA carries a longer share.
+// A chunk that ends inside a stream at slot a still reads slots a ..
+// kept[a-1], which the next chunk overwrites.  compact_stash_kernel copies
+// those slots aside before the compaction starts, and the chunk reads them
+// there.  Their number is at most the eviction's largest shift
+// kept[n-1] - (n-1); when that exceeds the stash, the per-stream units above
+// are used instead.
+//
 // A selection's eviction is compacted once: compact_consumed_kernel, launched
 // after the copy, sets each sequence's first moved slot to its length, so
 // another compaction before the next selection moves nothing.
@@ -51,16 +61,94 @@ constexpr int kMaxRPB = 32 * kMaxRowsPerLane;
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s: far beyond any real copy
 constexpr uint64_t kDrainNs = 100000000ull;   // 0.1 s per stage after a timeout
 
+#ifndef EPIKV_COMPACT_BALANCED
+#define EPIKV_COMPACT_BALANCED 1  // 0: per-stream units only
+#endif
 #ifndef EPIKV_COMPACT_STAGED_BLOCKS
 #define EPIKV_COMPACT_STAGED_BLOCKS 1024  // block-table entries kept in shared memory (larger tables: global reads)
 #endif
 constexpr int kStagedBlocks = EPIKV_COMPACT_STAGED_BLOCKS;
 
+constexpr int kStashThreads = 256;
+
+__host__ __device__ inline int list_ints(int n_seq) { return (n_seq + 31) / 32 * 32; }
+__host__ __device__ inline int pre_entries(int n_seq) { return (n_seq + 32) / 32 * 32; }
+
+// The batch entries that evicted, in batch order, into list; with pre, the
+// prefix sums of their moved rows per stream (pre[k] = rows of entries
+// before the k-th).  One warp; every CTA of both kernels builds the same.
+__device__ int evicting_entries(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
+                                int n_seq, int* list, int64_t* pre, int lane) {
+  int n_ev = 0;
+  int64_t acc = 0;
+  for (int base = 0; base < n_seq; base += 32) {
+    const int b = base + lane;
+    int len = 0;
+    if (b < n_seq) {
+      const int seq = seq_ids[b];
+      if (seq >= 0 && seq < dm.S) len = st.n_cache[seq] - st.first_changed[seq];
+    }
+    const bool ev = len > 0;
+    const unsigned m = __ballot_sync(0xffffffffu, ev);
+    int incl = ev ? len : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (ev) {
+      const int k = n_ev + __popc(m & ((1u << lane) - 1u));
+      list[k] = b;
+      if (pre) pre[k + 1] = acc + incl;
+    }
+    acc += __shfl_sync(0xffffffffu, incl, 31);
+    n_ev += __popc(m);
+  }
+  if (pre && lane == 0) pre[0] = 0;
+  __syncwarp();
+  return n_ev;
+}
+
+// Whether the balanced split applies: token budgets, a grid within the
+// stash's CTAs, and every evicting entry's largest shift (that of its last
+// kept slot) within one CTA's stash.
+__device__ bool balanced_split(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
+                               const int* list, int n_ev, const int32_t* __restrict__ kept, int kept_stride,
+                               int lane) {
+  if (!EPIKV_COMPACT_BALANCED || dm.layer_budgets || gridDim.x > kMaxStashCtas) return false;
+  bool ok = true;
+  for (int e = lane; e < n_ev; e += 32) {
+    const int b = list[e];
+    const int n = st.n_cache[seq_ids[b]];
+    ok = ok && __ldg(kept + (size_t)b * kept_stride + n - 1) - (n - 1) <= dm.stash_rows;
+  }
+  return __all_sync(0xffffffffu, ok);
+}
+
+// Entry e, stream q (layer * 2 + K|V) and row r (from the entry's first
+// moved slot) of row o of the balanced row space.
+__device__ __forceinline__ void locate_row(const int64_t* pre, int n_ev, int upe, int64_t o, int& e, int& q,
+                                           int64_t& r) {
+  int lo = 0, hi = n_ev - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (pre[mid] * upe <= o) lo = mid;
+    else hi = mid - 1;
+  }
+  e = lo;
+  const int64_t len = pre[e + 1] - pre[e];
+  const int64_t rel = o - pre[e] * upe;
+  q = (int)(rel / len);
+  r = rel - (int64_t)q * len;
+}
+
 struct Cursor {
-  int u;      // unit index (this CTA strides by gridDim.x)
+  int u;      // unit index (this CTA strides by gridDim.x); balanced: 0 while rows remain
   int i;      // next row of the unit
   int end;    // row past the last of the unit
   int b, seq, layer, kvk, hg;
+  int stash_at;   // balanced: sources at or past this slot are read from the next chunk's stash
+  int64_t o_end;  // balanced: row `end` in the balanced row space
 };
 
 template <bool kLayers>
@@ -72,39 +160,39 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   __shared__ char* dptr[kStages][kMaxRPB];
   __shared__ int stage_rows[kStages];
   int* list = reinterpret_cast<int*>(smem + kStages * kStageBytes);
-  int* bt_s = list + (n_seq + 31) / 32 * 32;  // the current sequence's block table
+  int64_t* pre = reinterpret_cast<int64_t*>(list + list_ints(n_seq));
+  int* bt_s = reinterpret_cast<int*>(pre + pre_entries(n_seq));  // the current sequence's block table
   const int lane = threadIdx.x;
 
   // ---- the batch entries that evicted (every CTA builds the same list)
-  int n_ev = 0;
-  for (int base = 0; base < n_seq; base += 32) {
-    const int b = base + lane;
-    bool ev = false;
-    if (b < n_seq) {
-      const int seq = seq_ids[b];
-      ev = seq >= 0 && seq < dm.S && st.first_changed[seq] < st.n_cache[seq];
-    }
-    const unsigned m = __ballot_sync(0xffffffffu, ev);
-    if (ev) list[n_ev + __popc(m & ((1u << lane) - 1u))] = b;
-    n_ev += __popc(m);
-  }
-  __syncwarp();
+  const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, kLayers ? nullptr : pre, lane);
   if (n_ev == 0) return;
+  const bool balanced = !kLayers && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, lane);
 
-  // ---- head split: whole token rows unless too few streams evict to give
-  // every CTA one (small TMA copies cost much more per byte than a tail)
+  // ---- per-stream units only: whole token rows unless too few streams
+  // evict to give every CTA one (small TMA copies cost much more per byte
+  // than a tail)
   const int G = gridDim.x;
   int hs = 1;
+  if (!balanced) {
 #if EPIKV_COMPACT_HEAD_SPLIT > 0
-  if (dm.H % EPIKV_COMPACT_HEAD_SPLIT == 0) hs = EPIKV_COMPACT_HEAD_SPLIT;
+    if (dm.H % EPIKV_COMPACT_HEAD_SPLIT == 0) hs = EPIKV_COMPACT_HEAD_SPLIT;
 #else
-  while ((long)n_ev * 2 * dm.L * hs < G && dm.H % (2 * hs) == 0 && (dm.H / (2 * hs)) * dm.d * 2 >= 256) hs *= 2;
+    while ((long)n_ev * 2 * dm.L * hs < G && dm.H % (2 * hs) == 0 && (dm.H / (2 * hs)) * dm.d * 2 >= 256) hs *= 2;
 #endif
+  }
   const int rb = (dm.H / hs) * dm.d * 2;               // bytes per row piece
   const int64_t piece_elems = (int64_t)(dm.H / hs) * dm.d;
   const int rpb = min(kStageBytes / rb, kMaxRPB);      // rows per batch
   const int upe = 2 * dm.L * hs;
-  const int units = n_ev * upe;
+  const int units = balanced ? 1 : n_ev * upe;
+  // balanced: this CTA's chunk [o_begin, o_stop) of the row space
+  int64_t o_begin = 0, o_stop = 0;
+  if (balanced) {
+    const int64_t total = pre[n_ev] * upe;
+    o_begin = (int64_t)blockIdx.x * total / G;
+    o_stop = (int64_t)(blockIdx.x + 1) * total / G;
+  }
   const bool paged = kv.layout == EPIKV_LAYOUT_PAGED;
   const bool bt_in_smem = paged && kv.max_blocks <= kStagedBlocks;
 
@@ -144,15 +232,42 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
         c.i = st.first_changed[c.seq];
         c.end = st.n_cache[c.seq];
       }
+      c.stash_at = INT_MAX;
       if (c.i < c.end) return;
       c.u = next_unit(c.u);
     }
   };
+  // balanced: the stream segment holding row o of the chunk
+  auto open_at = [&](Cursor& c, int64_t o) {
+    int e, q;
+    int64_t r;
+    locate_row(pre, n_ev, upe, o, e, q, r);
+    c.b = list[e];
+    c.seq = seq_ids[c.b];
+    c.layer = q >> 1;
+    c.kvk = q & 1;
+    c.hg = 0;
+    const int64_t rest = pre[e + 1] - pre[e] - r;       // rows of the stream from o on
+    c.i = st.first_changed[c.seq] + (int)r;
+    if (o_stop - o < rest) {                             // the chunk ends inside this stream
+      c.end = c.i + (int)(o_stop - o);
+      c.stash_at = c.end;
+    } else {
+      c.end = c.i + (int)rest;
+      c.stash_at = INT_MAX;
+    }
+    c.o_end = o + (c.end - c.i);
+  };
   auto advance = [&](Cursor& c) {
     c.i += rpb;
     if (c.i >= c.end) {
-      c.u = next_unit(c.u);
-      load_unit(c);
+      if (balanced) {
+        if (c.o_end < o_stop) open_at(c, c.o_end);
+        else c.u = units;
+      } else {
+        c.u = next_unit(c.u);
+        load_unit(c);
+      }
     }
   };
   // kept slots of the batch at c, one load per row, issued early and used later
@@ -203,11 +318,18 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
       if (r < nrows) {
         const int i = c.i + r;
         const int from = pk[j];
-        const int64_t so = from >= i ? slot_offset(c.layer, c.seq, from) : -1;
         const int64_t dof = slot_offset(c.layer, c.seq, i);
-        ok = so >= 0 && dof >= 0;
+        const char* from_ptr = nullptr;
+        if (from >= c.stash_at) {      // saved before the copy: the next chunk overwrites it
+          if (from - c.stash_at < dm.stash_rows)
+            from_ptr = st.stash + ((size_t)(blockIdx.x + 1) * dm.stash_rows + (from - c.stash_at)) * rb;
+        } else if (from >= i) {
+          const int64_t so = slot_offset(c.layer, c.seq, from);
+          if (so >= 0) from_ptr = kvb + (so + c.hg * piece_elems) * 2;
+        }
+        ok = from_ptr != nullptr && dof >= 0;
         if (ok) {
-          src[j] = kvb + (so + c.hg * piece_elems) * 2;
+          src[j] = from_ptr;
           dptr[s][r] = kvb + (dof + c.hg * piece_elems) * 2;
         } else {
           dptr[s][r] = nullptr;
@@ -227,8 +349,13 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   };
 
   Cursor ld;
-  ld.u = kLayers ? next_unit(0) : (int)blockIdx.x;
-  load_unit(ld);
+  if (balanced) {
+    ld.u = o_begin < o_stop ? 0 : units;
+    if (ld.u == 0) open_at(ld, o_begin);
+  } else {
+    ld.u = kLayers ? next_unit(0) : (int)blockIdx.x;
+    load_unit(ld);
+  }
   int pk[kMaxRowsPerLane];
   prefetch(ld, pk);
   int k_issue = 0, k_store = 0;
@@ -278,6 +405,60 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   }
 }
 
+// Before a balanced compaction: CTA g saves the slots that the chunk ending
+// where chunk g begins (slot a of its stream) reads from the region chunk g
+// overwrites, slots a .. kept[a-1], into stash g.  Nothing of the cache is
+// written, so every read sees the rows as the selection left them.
+__global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState st, Dims dm, KvDev kv,
+                                                                      const int32_t* __restrict__ seq_ids,
+                                                                      int n_seq, const int32_t* __restrict__ kept,
+                                                                      int kept_stride) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  int* list = reinterpret_cast<int*>(smem);
+  int64_t* pre = reinterpret_cast<int64_t*>(list + list_ints(n_seq));
+  __shared__ int s_nev, s_bal;
+  if (threadIdx.x < 32) {
+    const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, pre, threadIdx.x);
+    const bool bal = n_ev > 0 && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, threadIdx.x);
+    if (threadIdx.x == 0) {
+      s_nev = n_ev;
+      s_bal = bal;
+    }
+  }
+  __syncthreads();
+  if (!s_bal || blockIdx.x == 0) return;
+  const int n_ev = s_nev, upe = 2 * dm.L;
+  const int64_t total = pre[n_ev] * upe;
+  const int64_t o = (int64_t)blockIdx.x * total / gridDim.x;
+  if (o >= total) return;
+  int e, q;
+  int64_t r;
+  locate_row(pre, n_ev, upe, o, e, q, r);
+  if (r == 0) return;  // the chunk begins its stream: no other chunk reads its region
+  const int b = list[e], seq = seq_ids[b];
+  const int a = st.first_changed[seq] + (int)r;
+  const int x = __ldg(kept + (size_t)b * kept_stride + a - 1) - a + 1;
+  if (x <= 0) return;
+  if (x > dm.stash_rows) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_KEPT);
+    return;
+  }
+  const int layer = q >> 1;
+  const char* kvb = (q & 1) ? kv.base[1] : kv.base[0];
+  const int v16 = dm.H * dm.d / 8;  // 16-byte vectors per row
+  uint4* dst = reinterpret_cast<uint4*>(st.stash + (size_t)blockIdx.x * dm.stash_rows * dm.H * dm.d * 2);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  for (int row = warp; row < x; row += kStashThreads / 32) {
+    const int64_t so = kv_row_offset(kv, layer, seq, a + row, dm.T);
+    if (so < 0) {
+      if (lane == 0) set_error(st.err, EPIKV_DEV_SLOT);
+      continue;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(kvb + so * 2);
+    for (int k = lane; k < v16; k += 32) dst[(size_t)row * v16 + k] = __ldg(src + k);
+  }
+}
+
 // The batch entries' evictions have been applied: nothing is left pending.
 __global__ void compact_consumed_kernel(DevState st, Dims dm, const int32_t* __restrict__ seq_ids, int n_seq) {
   for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < n_seq; b += gridDim.x * blockDim.x) {
@@ -291,9 +472,12 @@ __global__ void compact_consumed_kernel(DevState st, Dims dm, const int32_t* __r
 
 static int g_ctas_per_sm = 0;
 
+static size_t stash_smem(int n_seq) {
+  return (size_t)list_ints(n_seq) * sizeof(int) + (size_t)pre_entries(n_seq) * sizeof(int64_t);
+}
+
 static size_t compact_smem(int n_seq) {
-  return (size_t)kStages * kStageBytes + (size_t)((n_seq + 31) / 32 * 32) * sizeof(int) +
-         (size_t)kStagedBlocks * sizeof(int);
+  return (size_t)kStages * kStageBytes + stash_smem(n_seq) + (size_t)kStagedBlocks * sizeof(int);
 }
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm) {
@@ -303,6 +487,9 @@ cudaError_t compact_prepare(int device, int* ctas_per_sm) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(compact_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)compact_smem(4096));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(compact_stash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)stash_smem(4096));
   if (e != cudaSuccess) return e;
   int n = 0;
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel<false>, 32, compact_smem(64));
@@ -317,12 +504,21 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
                            const int32_t* kept, int kept_stride, const KvDev& kv, int ctas,
                            cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
-  if (dm.layer_budgets)
+  cudaError_t e = cudaSuccess;
+  if (dm.layer_budgets) {
     compact_kernel<true><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
-  else
+  } else {
+    if (ctas <= kMaxStashCtas) {  // the balanced split's stash (the kernel checks whether it applies)
+      compact_stash_kernel<<<ctas, kStashThreads, stash_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept,
+                                                                              kept_stride);
+      ++*launches;
+      e = cudaGetLastError();
+      if (e != cudaSuccess) return e;
+    }
     compact_kernel<false><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  }
   ++*launches;
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   compact_consumed_kernel<<<(n_seq + 255) / 256, 256, 0, stream>>>(st, dm, seq_ids, n_seq);
   ++*launches;
