@@ -476,7 +476,7 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src,
                      "traffic": traffic, "algorithmic_bytes_per_launch": compact_bytes / args.steps},
-        "gpu_launches": 5 * args.steps,   # Lag-KV partial, finalize, select, compaction, eviction consumed
+        "gpu_launches": 6 * args.steps,   # Lag-KV partial, finalize, select, stash, compaction, eviction consumed
         "clocks": clk,
         "e2e": e2e,
     }
@@ -582,7 +582,7 @@ def run_bandz2k(args):
             "roofline": {"bound": "hbm", "kernel": "score phase (bandz_g_kernel + score_finalize_kernel)",
                          "achieved": g, "peak": peak, "unit": "GB/s", "frac": g / peak, "peak_source": peak_src,
                          "traffic": None, "algorithmic_bytes_per_launch": score_bytes},
-            "gpu_launches": 6 * args.steps}   # reset, g, finalize, select, compaction, eviction consumed
+            "gpu_launches": 7 * args.steps}   # reset, g, finalize, select, stash, compaction, eviction consumed
     print(json.dumps(line), flush=True)
 
 
@@ -1025,7 +1025,8 @@ def run_window(args):
                          "frac": ach / peak, "peak_source": peak_src, "traffic": None,
                          "algorithmic_bytes_per_launch": compact_bytes / n_launch,
                          "timing": "eager calls, phase events"},
-            "gpu_launches": (6 if wl.kinds & E.EPIKV_SCORE_LAGKV else 5) * n_launch,
+            # g, [Lag-KV partial,] finalize, select, stash, compaction, eviction consumed
+            "gpu_launches": (7 if wl.kinds & E.EPIKV_SCORE_LAGKV else 6) * n_launch,
             "clocks": clk}
     print(json.dumps(line), flush=True)
 

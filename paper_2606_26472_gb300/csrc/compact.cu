@@ -69,7 +69,8 @@ constexpr uint64_t kDrainNs = 100000000ull;   // 0.1 s per stage after a timeout
 #endif
 constexpr int kStagedBlocks = EPIKV_COMPACT_STAGED_BLOCKS;
 
-constexpr int kStashThreads = 256;
+constexpr int kStashThreads = 512;
+constexpr int kStashUnroll = 4;
 
 __host__ __device__ inline int list_ints(int n_seq) { return (n_seq + 31) / 32 * 32; }
 __host__ __device__ inline int pre_entries(int n_seq) { return (n_seq + 32) / 32 * 32; }
@@ -447,15 +448,35 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   const char* kvb = (q & 1) ? kv.base[1] : kv.base[0];
   const int v16 = dm.H * dm.d / 8;  // 16-byte vectors per row
   uint4* dst = reinterpret_cast<uint4*>(st.stash + (size_t)blockIdx.x * dm.stash_rows * dm.H * dm.d * 2);
+  // each warp copies two rows at a time, every lane's loads issued before its stores
+  constexpr int kWarps = kStashThreads / 32;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  for (int row = warp; row < x; row += kStashThreads / 32) {
-    const int64_t so = kv_row_offset(kv, layer, seq, a + row, dm.T);
-    if (so < 0) {
-      if (lane == 0) set_error(st.err, EPIKV_DEV_SLOT);
-      continue;
+  for (int r0 = warp; r0 < x; r0 += 2 * kWarps) {
+    const int r1 = r0 + kWarps;
+    const int64_t s0 = kv_row_offset(kv, layer, seq, a + r0, dm.T);
+    const int64_t s1 = r1 < x ? kv_row_offset(kv, layer, seq, a + r1, dm.T) : -2;
+    if ((s0 == -1 || s1 == -1) && lane == 0) set_error(st.err, EPIKV_DEV_SLOT);
+    const uint4* p0 = reinterpret_cast<const uint4*>(kvb + s0 * 2);
+    const uint4* p1 = reinterpret_cast<const uint4*>(kvb + s1 * 2);
+    for (int k0 = lane; k0 < v16; k0 += kStashUnroll * 32) {
+      uint4 v0[kStashUnroll], v1[kStashUnroll];
+#pragma unroll
+      for (int u = 0; u < kStashUnroll; ++u) {
+        const int k = k0 + 32 * u;
+        if (k < v16) {
+          if (s0 >= 0) v0[u] = __ldg(p0 + k);
+          if (s1 >= 0) v1[u] = __ldg(p1 + k);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kStashUnroll; ++u) {
+        const int k = k0 + 32 * u;
+        if (k < v16) {
+          if (s0 >= 0) dst[(size_t)r0 * v16 + k] = v0[u];
+          if (s1 >= 0) dst[(size_t)r1 * v16 + k] = v1[u];
+        }
+      }
     }
-    const uint4* src = reinterpret_cast<const uint4*>(kvb + so * 2);
-    for (int k = lane; k < v16; k += 32) dst[(size_t)row * v16 + k] = __ldg(src + k);
   }
 }
 
