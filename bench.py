@@ -50,9 +50,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    # host-to-device copies share the machine's host memory path: over ~1 s a
-    # burst of slow copies on the shared host costs a few percent, not half
-    p.add_argument("--e2e-steps", type=int, default=100)
+    # end-to-end steps, each with its own 512 MiB of new K/V in pinned host memory
+    p.add_argument("--e2e-steps", type=int, default=50)
     # CTAs of the end-to-end measurement's host-to-device upload kernel
     p.add_argument("--upload-ctas", type=int, default=32)
     # a scaled-down variant of the same workload, for profiler captures
@@ -382,15 +381,17 @@ def run_ours(args):
         # stream while step i runs, as a serving loop would overlap them
         tabs = [table(e2e_base + j * Bn * fresh) for j in range(2)]
         views_e = [cache.view(t) for t in tabs]
-        n_payload = min(4, e2e_steps)
-        payload = torch.empty((n_payload, 2, L, Bn * fresh, bs, H, d), dtype=torch.bfloat16, pin_memory=True)
+        # every step's own new tokens (fresh positions, as in the timed loop),
+        # one pinned buffer per step
+        payload = [torch.empty((2, L, Bn * fresh, bs, H, d), dtype=torch.bfloat16, pin_memory=True)
+                   for _ in range(e2e_steps)]
         pos_base = K + n_steps * C
         lo = e2e_base
-        for j in range(n_payload):
+        for j in range(e2e_steps):
             for b in range(Bn):
                 dt.kv(b, pos_base + j * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tabs[0]))
-            payload[j, 0].copy_(cache.k[:, lo:lo + Bn * fresh])
-            payload[j, 1].copy_(cache.v[:, lo:lo + Bn * fresh])
+            payload[j][0].copy_(cache.k[:, lo:lo + Bn * fresh])
+            payload[j][1].copy_(cache.v[:, lo:lo + Bn * fresh])
         lens = torch.empty((e2e_steps, Bn), dtype=torch.int32, pin_memory=True)
         copy_stream = torch.cuda.Stream(device=dev)
         copied = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
@@ -412,7 +413,7 @@ def run_ours(args):
             if i >= 2:
                 copy_stream.wait_event(stepped[i - 2])
             copy_start[i].record(copy_stream)
-            src = payload[i % n_payload]
+            src = payload[i]
             for kind, pool in ((0, cache.k), (1, cache.v)):
                 upload_2d(pool[0, lo_i].data_ptr(), pitch, src[kind].data_ptr(), plane, plane, L, up_ctas, copy_stream)
             copied[i].record(copy_stream)
@@ -420,6 +421,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
+        stats_e0 = E.epikv_get_stats(ctx)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
@@ -447,7 +449,8 @@ def run_ours(args):
                "median_ms": {"h2d_copy": copy_ms[len(copy_ms) // 2], "step": step_ms[len(step_ms) // 2],
                              "wall_per_step": e_ms / e2e_steps},
                "max_ms": {"h2d_copy": copy_ms[-1], "step": step_ms[-1]},
-               "slow_copies": sum(c > 2 * copy_ms[len(copy_ms) // 2] for c in copy_ms)}
+               "slow_copies": sum(c > 2 * copy_ms[len(copy_ms) // 2] for c in copy_ms),
+               "rows_moved_per_step": (E.epikv_get_stats(ctx)["rows_moved"] - stats_e0["rows_moved"]) / e2e_steps}
         st_, code = E.epikv_get_error(ctx)
         assert st_ == E.EPIKV_OK, f"device error {code} in e2e"
 
@@ -469,6 +472,7 @@ def run_ours(args):
                    "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
         "compaction_gbs": ach,
+        "rows_moved_per_step": rows_moved / args.steps,
         "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
                                 "compact": t_compact / args.steps},
         "compact_ms_min_median_max": [per_compact[0], per_compact[len(per_compact) // 2], per_compact[-1]],
