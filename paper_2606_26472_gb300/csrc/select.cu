@@ -97,12 +97,61 @@ __device__ __forceinline__ int block_min(int v, int* sh) {
 
 // Slot j <- slot kept[j] of the sequence's scores (every kind) and positions,
 // for j from fe to n_kept, in place: safe in increasing j because kept[j] >= j
-// and each round reads all its sources before any of its stores.  Every
-// thread of the block calls it.
+// and each round reads all its sources before any of its stores.  A round
+// stages as many rows as `stage` (stage_words 32-bit words of shared memory,
+// free by now) holds, all their loads in flight together; without room for
+// a round of kSelThreads rows, a round is one row per thread in registers.
+// Every thread of the block calls it.
 __device__ __forceinline__ void compact_metadata(const DevState& st, const Dims& dm, int seq,
-                                                 const int32_t* __restrict__ kept, int fe, int n_kept) {
+                                                 const int32_t* __restrict__ kept, int fe, int n_kept,
+                                                 uint32_t* stage, int stage_words) {
   const int tid = threadIdx.x;
   int32_t* ps = st.pos + (size_t)seq * dm.T;
+  const size_t base = (size_t)seq * dm.T;
+  unsigned on = 0;  // the score kinds held
+#pragma unroll
+  for (int k = 0; k < kNumKinds; ++k) on |= (st.score[k] != nullptr ? 1u : 0u) << k;
+  const int n_on = __popc(on);
+  const int cap = stage_words / (n_on + 1);
+  if (cap >= kSelThreads) {
+    constexpr int U = 4;  // rows per thread with their loads in flight together
+    for (int j0 = fe; j0 < n_kept; j0 += cap) {
+      const int m = min(cap, n_kept - j0);
+      for (int r0 = tid; r0 < m; r0 += U * kSelThreads) {
+        int src[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) src[u] = r0 + u * kSelThreads < m ? kept[j0 + r0 + u * kSelThreads] : -1;
+        uint32_t v[U][kNumKinds + 1];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          if (src[u] < 0) continue;
+#pragma unroll
+          for (int k = 0; k < kNumKinds; ++k)
+            if (on >> k & 1u) v[u][k] = __float_as_uint(st.score[k][base + src[u]]);
+          v[u][kNumKinds] = (uint32_t)ps[src[u]];
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          if (src[u] < 0) continue;
+          const int r = r0 + u * kSelThreads;
+#pragma unroll
+          for (int k = 0; k < kNumKinds; ++k)
+            if (on >> k & 1u) stage[__popc(on & ((1u << k) - 1u)) * cap + r] = v[u][k];
+          stage[n_on * cap + r] = v[u][kNumKinds];
+        }
+      }
+      __syncthreads();
+      for (int r = tid; r < m; r += kSelThreads) {
+        int q = 0;
+#pragma unroll
+        for (int k = 0; k < kNumKinds; ++k)
+          if (st.score[k]) st.score[k][base + j0 + r] = __uint_as_float(stage[(q++) * cap + r]);
+        ps[j0 + r] = (int32_t)stage[n_on * cap + r];
+      }
+      __syncthreads();
+    }
+    return;
+  }
   for (int j0 = fe; j0 < n_kept; j0 += kSelThreads) {
     const int j = j0 + tid;
     float v[kNumKinds];
@@ -193,7 +242,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
                                                              const int32_t* __restrict__ budget,
                                                              const int32_t* __restrict__ trigger,
                                                              int32_t* __restrict__ kept_out, int kept_stride,
-                                                             int32_t* __restrict__ n_kept_out, int staged_cap) {
+                                                             int32_t* __restrict__ n_kept_out, int staged_cap,
+                                                             int smem_words) {
   const int b = blockIdx.x, tid = threadIdx.x;
   const int seq = seq_ids[b];
   if (seq < 0 || seq >= dm.S) {
@@ -306,8 +356,9 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   const int fe = min(block_min(first_ev, sh_scan), n_kept);
   __syncthreads();  // kept list visible to the whole block
 
-  // ---- compact slot metadata in place (kept[i] >= i, increasing i)
-  compact_metadata(st, dm, seq, out, fe, n_kept);
+  // ---- compact slot metadata in place (kept[i] >= i, increasing i); the
+  // staged keys are no longer needed, so their shared memory stages it
+  compact_metadata(st, dm, seq, out, fe, n_kept, skey, smem_words);
   if (tid == 0) {
     st.n_cache[seq] = n_kept;
     st.first_changed[seq] = fe;
@@ -510,7 +561,7 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
                                                                   const int32_t* __restrict__ seq_ids,
                                                                   const int32_t* __restrict__ budget,
                                                                   const int32_t* __restrict__ trigger,
-                                                                  int kept_stride) {
+                                                                  int kept_stride, int smem_words) {
   constexpr int NW = kSelThreads / 32;
   const int b = blockIdx.x, tid = threadIdx.x, L = dm.L;
   const int lane = tid & 31;
@@ -567,7 +618,8 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
   }
   fe = min(block_min(fe, sh_scan), n_union);
   __syncthreads();  // the union's kept list is visible to the whole block
-  compact_metadata(st, dm, seq, mkept, fe, n_union);
+  extern __shared__ uint32_t stage[];
+  compact_metadata(st, dm, seq, mkept, fe, n_union, stage, smem_words);
   // every new mask lands in its slot (the slots before fe did not move)
   for (int j = tid; j < n_union; j += kSelThreads) mk[j] = mn[mkept[j]];
   if (tid == 0) {
@@ -579,14 +631,22 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
 }
 
 // Candidate keys staged in shared memory: caches of up to kSelStagedMax slots.
-constexpr int kSelStagedMax = 48 * 1024;  // 192 KiB of u32 keys
+// The same memory then stages the slot metadata's compaction: one round for
+// every kind's score and the position of each slot, when it fits.
+constexpr int kSelStagedMax = 48 * 1024;  // 192 KiB of u32 words
 static int sel_staged_cap(const Dims& dm) { return dm.T <= kSelStagedMax ? dm.T : 0; }
-static size_t sel_smem(const Dims& dm) { return (size_t)sel_staged_cap(dm) * sizeof(uint32_t); }
+static int sel_smem_words(const Dims& dm) {
+  const int64_t meta = (int64_t)(__builtin_popcount((unsigned)dm.kinds) + 1) * dm.T;
+  const int64_t w = meta > sel_staged_cap(dm) ? meta : sel_staged_cap(dm);
+  return (int)(w < kSelStagedMax ? w : kSelStagedMax);
+}
+static size_t sel_smem(const Dims& dm) { return (size_t)sel_smem_words(dm) * sizeof(uint32_t); }
 
 cudaError_t select_prepare() {
   const int mx = kSelStagedMax * (int)sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(select_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(layer_union_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
   return e;
 }
 
@@ -600,13 +660,16 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ++*launches;
-    layer_union_kernel<<<n_seq, kSelThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept_stride);
+    layer_union_kernel<<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept_stride,
+                                                                     sel_smem_words(dm));
   } else if (dm.select_chunk > 1)
     select_kernel<true><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
-                                                                      kept_stride, n_kept, sel_staged_cap(dm));
+                                                                      kept_stride, n_kept, sel_staged_cap(dm),
+                                                                      sel_smem_words(dm));
   else
     select_kernel<false><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
-                                                                       kept_stride, n_kept, sel_staged_cap(dm));
+                                                                       kept_stride, n_kept, sel_staged_cap(dm),
+                                                                       sel_smem_words(dm));
   ++*launches;
   return cudaGetLastError();
 }
