@@ -291,30 +291,25 @@ __device__ __forceinline__ void transpose_sum(float (&v)[NV], int lane) {
 // computed two channels per instruction (f32x2); the segment's 2 x 8 moments
 // are summed over the head's lanes by one transposed reduction into shared
 // memory, where a thread per token forms each head's variance.
-template <int LH>
-__global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
-                                                             const int32_t* __restrict__ seq_ids,
-                                                             const int32_t* __restrict__ cu_new,
-                                                             int max_new) {
-  const int b = blockIdx.y;
-  const int seq = seq_ids[b];
-  const int n_new = cu_new[b + 1] - cu_new[b];
-  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
-    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
-    return;
-  }
-  const int layer = blockIdx.x >> 1, kvk = blockIdx.x & 1;
-  const int tid = threadIdx.x;
+//
+// The stream's work is lag_stream, which the one-token decode kernel
+// (token_kernel) runs unchanged for its K/V CTAs.
+// SEG is the longest segment: kLagSeg, or 1 for one-token calls (fewer
+// registers; the reductions pair lanes in the same order either way, so the
+// sums are the same bit for bit).  With HALF, each half of a 256-thread
+// block runs its own stream (K in the first half, V in the second; H*d/8 <=
+// 128), with its own shared memory.
+template <int LH, int SEG = kLagSeg, bool HALF = false>
+__device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, const KvDev& kv, int seq,
+                                           int n_new, int layer, int kvk, int nc0) {
+  const int stream = layer * 2 + kvk;  // this stream's column of the per-token partials
+  const int tid = HALF ? (int)(threadIdx.x & 127) : (int)threadIdx.x;
+  const int nthr = HALF ? 128 : (int)blockDim.x;
+  const int half = HALF ? kvk : 0;
   const int h = tid / LH, q = tid % LH;
   const bool active = h < dm.H;
   const int hd = dm.H * dm.d;
-  // the new rows' first slot: this layer's own length under per-layer budgets
-  const int nc0 = dm.layer_budgets ? st.n_layer[seq * dm.L + layer] : st.n_cache[seq];
   const int p0 = st.n_seen[seq];
-  if (nc0 + n_new > dm.T) {
-    if (tid == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
-    return;
-  }
   const int ch = h * dm.d + q * 8;  // first channel of this thread within the token row
   const bool need_norm = dm.kinds & kNormKinds;   // uniform across the grid
   const bool need_raw = dm.kinds & kRawKinds;
@@ -332,10 +327,13 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
 
   const float inv_d = 1.f / (float)dm.d;
   const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
-  __shared__ int64_t soff[kLagOffs];
-  constexpr int NV = 2 * kLagSeg;      // moments of a segment: (sum y, sum y^2) per token
-  __shared__ float red[2][32][NV];      // [segment parity][head][moment]; the host admits H <= 32
-  __shared__ float hr[2][kLagSeg][32];  // raw variances, same layout
+  __shared__ int64_t soff_s[HALF ? 2 : 1][kLagOffs];
+  constexpr int NV = 2 * SEG;      // moments of a segment: (sum y, sum y^2) per token
+  __shared__ float red_s[HALF ? 2 : 1][2][32][NV];  // [half][segment parity][head][moment]; the host admits H <= 32
+  __shared__ float hr_s[HALF ? 2 : 1][2][SEG][32];  // raw variances, same layout
+  int64_t* soff = soff_s[half];
+  float (*red)[32][NV] = red_s[half];
+  float (*hr)[SEG][32] = hr_s[half];
   float* part = need_norm ? st.lag_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
   float* rpart = need_raw ? st.raw_part + (size_t)seq * dm.max_new * (2 * dm.L) : nullptr;
   int r = p0 % dm.lag;                   // position of the next token inside its chunk
@@ -344,14 +342,14 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
   for (int g0 = 0; g0 < n_new; g0 += kLagOffs) {
     const int gn = min(kLagOffs, n_new - g0);
     __syncthreads();
-    for (int t = tid; t < gn; t += blockDim.x) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
+    for (int t = tid; t < gn; t += nthr) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
     __syncthreads();
     for (int i = 0; i < gn;) {
-      const int seg = min(min(dm.lag - r, gn - i), kLagSeg);
+      const int seg = min(min(dm.lag - r, gn - i), SEG);
       const bool has_prev = p0 + g0 + i >= dm.lag;   // the segment's chunk is not chunk 0
-      uint4 x[kLagSeg];
+      uint4 x[SEG];
 #pragma unroll
-      for (int j = 0; j < kLagSeg; ++j) {
+      for (int j = 0; j < SEG; ++j) {
         x[j] = make_uint4(0, 0, 0, 0);
         if (j < seg && active) {
           const int64_t off = soff[i + j];
@@ -362,7 +360,7 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
         }
       }
 #pragma unroll
-      for (int j = 0; j < kLagSeg; ++j) {
+      for (int j = 0; j < SEG; ++j) {
         if (j < seg) {
           if (need_raw) {  // population variance of the stored vector over the head dimension
             float xf[8], s1 = 0.f;
@@ -384,7 +382,7 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
       if (has_prev && need_norm) {  // uniform across the block
         float v[NV];
 #pragma unroll
-        for (int j = 0; j < kLagSeg; ++j) {
+        for (int j = 0; j < SEG; ++j) {
           v[2 * j] = v[2 * j + 1] = 0.f;
           if (j < seg) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
         }
@@ -404,7 +402,7 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
         cmx = x[0];
       }
 #pragma unroll
-      for (int j = 0; j < kLagSeg; ++j)
+      for (int j = 0; j < SEG; ++j)
         if (j < seg) {
           cmn = q_min(cmn, x[j]);
           cmx = q_max(cmx, x[j]);
@@ -418,12 +416,12 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
               const float mean = red[parity][hh][2 * tid] * inv_d;
               sum += fmaxf(fmaf(-mean, mean, red[parity][hh][2 * tid + 1] * inv_d), 0.f);
             }
-          part[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+          part[(size_t)(g0 + i + tid) * (2 * dm.L) + stream] = sum;
         }
         if (need_raw) {
           float sum = 0.f;
           for (int hh = 0; hh < dm.H; ++hh) sum += hr[parity][tid][hh];
-          rpart[(size_t)(g0 + i + tid) * (2 * dm.L) + blockIdx.x] = sum;
+          rpart[(size_t)(g0 + i + tid) * (2 * dm.L) + stream] = sum;
         }
       }
       parity ^= 1;
@@ -443,6 +441,28 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
     *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = cmn;
     *reinterpret_cast<uint4*>(rng + 3 * hd + ch) = cmx;
   }
+}
+
+template <int LH>
+__global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
+                                                             const int32_t* __restrict__ seq_ids,
+                                                             const int32_t* __restrict__ cu_new,
+                                                             int max_new) {
+  const int b = blockIdx.y;
+  const int seq = seq_ids[b];
+  const int n_new = cu_new[b + 1] - cu_new[b];
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > max_new) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int layer = blockIdx.x >> 1, kvk = blockIdx.x & 1;
+  // the new rows' first slot: this layer's own length under per-layer budgets
+  const int nc0 = dm.layer_budgets ? st.n_layer[seq * dm.L + layer] : st.n_cache[seq];
+  if (nc0 + n_new > dm.T) {
+    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+    return;
+  }
+  lag_stream<LH>(st, dm, kv, seq, n_new, layer, kvk, nc0);
 }
 
 #ifndef EPIKV_FIN_TILE
@@ -614,45 +634,24 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
 }
 
 
-// One new token per sequence with the band kinds only (a decode step):
-// g and the rolling z-score in one launch.  grid (band layers, batch
-// entries), kGThreads threads: each CTA forms its band row's g exactly as
-// bandz_g_kernel does (same per-thread vectors, warp sums and fixed-order
-// cross-warp sum) and writes the ring and h_prev; the last CTA of a sequence
-// (atomic ticket after a fence; no CTA waits) stages every band's window from
-// the ring in shared memory -- the earlier positions' g are the per-sequence
-// running state -- and forms z and the score exactly as score_finalize_kernel
-// does (a lane per band, the same shifted two-pass, the same butterfly over
-// the lanes), then commits the sequence's counters.  Results equal the
-// two-kernel path bit for bit.
+// ---- one new token per sequence (a decode step)
+#ifndef EPIKV_TOKEN_MINB
+// token_kernel CTAs resident per SM: 5 caps registers at 48 (64 ragged
+// sequences' decode step: 45.7 / 41.1 / 38.5 / 38.5 us at 3 / 4 / 5 / 6)
+#define EPIKV_TOKEN_MINB 5
+#endif
+//
+// The band g of one (band layer, sequence): the new row against the previous
+// one (h_prev), exactly as bandz_g_kernel forms it (same per-thread vectors,
+// warp sums and fixed-order cross-warp sum); writes the ring and h_prev.
+// Every thread of a kGThreads block calls it.
 template <int VPT>
-__global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dims dm, BandRows rows,
-                                                                 int64_t row_stride,
-                                                                 const int32_t* __restrict__ seq_ids,
-                                                                 const int32_t* __restrict__ cu_new) {
-  const int band = blockIdx.x, b = blockIdx.y;
+__device__ __forceinline__ void band_token_g(const DevState& st, const Dims& dm, const BandRows& rows,
+                                             int64_t row_stride, int band, int seq, int r0, int pos, int par) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int seq = seq_ids[b];
-  const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
-  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > 1 || cu_new[0] != 0) {
-    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_BATCH);
-    return;
-  }
-  if (n_new == 0) return;
   const int nb = dm.nA + dm.nB;
-  const int nc0 = st.n_cache[seq];
-  const int pos = st.n_seen[seq];
-  if (nc0 + 1 > dm.T) {
-    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
-    return;
-  }
-  const int par = st.hp_parity[seq];
   const int VR = dm.D >> 3;
-  const int Gm = dm.G - 1;
   __shared__ float red[kGThreads / 32];
-  __shared__ int s_last;
-
-  // ---- g of this band layer (the row against the previous one, h_prev)
   const __nv_bfloat16* cur = rows.p[band] + (int64_t)r0 * row_stride;
   const __nv_bfloat16* prow = st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D;
   __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
@@ -687,78 +686,230 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
     float sum = 0.f;
 #pragma unroll
     for (int w = 0; w < kGThreads / 32; ++w) sum += red[w];
-    if (pos >= 1) st.g_ring[((size_t)seq * nb + band) * dm.G + (pos & Gm)] = sqrtf(sum);
+    if (pos >= 1) st.g_ring[((size_t)seq * (dm.nA + dm.nB) + band) * dm.G + (pos & (dm.G - 1))] = sqrtf(sum);
+  }
+}
+
+// The band kinds' scores of the new token at slot nc0: every band's window
+// staged from the ring in `win` ([nb][z_window] floats of shared memory; the
+// earlier positions' g are the per-sequence running state), then z and the
+// band combination exactly as score_finalize_kernel forms them (a lane per
+// band, the same shifted two-pass, the same butterfly over the lanes).
+// Every thread of the block calls it; warp 0 writes.
+__device__ __forceinline__ void band_token_scores(const DevState& st, const Dims& dm, int seq, int nc0, int pos,
+                                                  float* win) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nb = dm.nA + dm.nB;
+  const int Gm = dm.G - 1;
+  const int w = dm.z_window;
+  const int n = pos >= 1 ? min(w, pos) : 0;
+  for (int idx = tid; idx < nb * n; idx += blockDim.x) {
+    const int bb = idx / n, k = idx - bb * n;
+    win[bb * w + k] = __ldcg(st.g_ring + ((size_t)seq * nb + bb) * dm.G + ((pos - k) & Gm));
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  const int lpt = nb <= 16 ? 16 : 32;  // the lanes of one token, as in score_finalize_kernel
+  const int bl = lane % lpt;
+  const bool live = lane < lpt && pos >= 1 && bl < nb;
+  float za = 0.f, zb = 0.f, ma = 0.f, mb = 0.f;
+  if (live) {
+    const float* row = win + bl * w;  // row[k] = g at position pos - k
+    if (dm.kinds & EPIKV_SCORE_BANDZ) {
+      const float gnew = row[0];
+      float dsum = 0.f;
+      for (int k = 0; k < n; ++k) dsum += row[k] - gnew;
+      const float mean_d = dsum / (float)n;
+      float dev = 0.f;
+      for (int k = 0; k < n; ++k) {
+        const float e = (row[k] - gnew) - mean_d;
+        dev = fmaf(e, e, dev);
+      }
+      const float sigma = sqrtf(dev / (float)n);
+      const float z = -mean_d / (sigma + dm.z_eps);
+      if (bl < dm.nA) za = z; else zb = z;
+    }
+    if (dm.kinds & EPIKV_SCORE_HSVAR) {
+      float sum = 0.f;
+      for (int k = 0; k < n; ++k) sum += row[k];
+      const float gbar = sum / (float)n;
+      if (bl < dm.nA) ma = gbar; else mb = gbar;
+    }
+  }
+  for (int o = lpt >> 1; o > 0; o >>= 1) {
+    za += __shfl_xor_sync(0xffffffffu, za, o);
+    zb += __shfl_xor_sync(0xffffffffu, zb, o);
+    ma += __shfl_xor_sync(0xffffffffu, ma, o);
+    mb += __shfl_xor_sync(0xffffffffu, mb, o);
+  }
+  if (lane == 0) {
+    const size_t slot = (size_t)seq * dm.T + nc0;
+    if (dm.kinds & EPIKV_SCORE_BANDZ) st.score[0][slot] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
+    if (dm.kinds & EPIKV_SCORE_HSVAR) st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
+  }
+}
+
+// The K/V kinds' scores of the new token at slot nc0 (position pos), exactly
+// as score_finalize_kernel forms them for a call's single token: u from the
+// per-(layer, K|V) partials the stream CTAs wrote, summed in stream order by
+// one thread (the warp first loads them into shared memory together, so the
+// sum waits on one round of loads, not on 2L); its rolling mean over this u
+// and the ring's earlier ones, a lane per window position in the same order,
+// the same warp sum.  Warp 0 calls it.
+__device__ __forceinline__ void kv_token_scores(const DevState& st, const Dims& dm, int seq, int nc0, int pos) {
+  const int lane = threadIdx.x & 31;
+  __shared__ float pv[2 * 64];  // the host admits at most 64 layers
+  const int Gm = dm.G - 1;
+  const int w = dm.lag_window;
+  const int n = min(w, pos + 1);
+  const float inv_lh = 1.f / (float)(dm.L * dm.H);
+  for (int qk = 0; qk < 4; ++qk) {
+    const int kind = kv_kind(qk);
+    if (!(dm.kinds & kind)) continue;
+    const bool raw = kind & kRawKinds;
+    const float* part = (raw ? st.raw_part : st.lag_part) + (size_t)seq * dm.max_new * (2 * dm.L);
+    const int q0 = kind == EPIKV_SCORE_KVVAL ? 1 : 0;
+    const int qs = kind == EPIKV_SCORE_LAGKV ? 1 : 2;
+    float* ring = st.u_ring[qk] + (size_t)seq * dm.G;
+    float u = 0.f;
+    if (raw || pos >= dm.lag) {  // the normalised kinds have no value in chunk 0
+      for (int q = lane; q < 2 * dm.L; q += 32) pv[q] = __ldcg(part + q);
+      __syncwarp();
+      if (lane == 0) {
+        float s = 0.f;
+        for (int q = q0; q < 2 * dm.L; q += qs) s += pv[q];
+        u = s * inv_lh;
+      }
+      __syncwarp();  // pv is reused kind after kind
+    }
+    u = __shfl_sync(0xffffffffu, u, 0);
+    float acc = 0.f;
+    for (int k = lane; k < n; k += 32) acc += k == 0 ? u : __ldcg(ring + ((pos - k) & Gm));
+    const float mean = warp_sum(acc) / (float)n;
+    if (lane == 0) {
+      st.score[kind_index(kind)][(size_t)seq * dm.T + nc0] = mean;
+      ring[pos & Gm] = u;
+    }
+  }
+}
+
+// The decode step's commit of one sequence (as score_finalize_kernel's last
+// CTA does it): the new slot's position, the counters, h_prev's parity.
+// One thread.
+__device__ __forceinline__ void token_commit(const DevState& st, const Dims& dm, int seq, int nc0, int pos) {
+  const size_t slot = (size_t)seq * dm.T + nc0;
+  st.pos[slot] = pos;
+  if (dm.layer_budgets) {  // the new token is in every layer
+    st.lmask[slot] = dm.L == 64 ? ~0ull : (1ull << dm.L) - 1ull;
+    for (int l = 0; l < dm.L; ++l) {
+      st.n_layer[seq * dm.L + l] += 1;
+      st.lfirst[seq * dm.L + l] = st.n_layer[seq * dm.L + l];
+    }
+  }
+  if (st.first_changed[seq] < nc0) set_error(st.err, EPIKV_DEV_KEPT);
+  st.first_changed[seq] = nc0 + 1;
+  st.n_cache[seq] = nc0 + 1;
+  st.n_seen[seq] = pos + 1;
+  if (dm.kinds & kBandKinds) st.hp_parity[seq] ^= 1;
+  atomicAdd(&st.stats[0], 1ull);
+  st.ticket[seq] = 0u;
+}
+
+// One new token per sequence with the band kinds only: g and the rolling
+// z-score in one launch.  grid (band layers, batch entries), kGThreads
+// threads: each CTA forms its band row's g (band_token_g); the last CTA of a
+// sequence (atomic ticket after a fence; no CTA waits) forms the scores
+// (band_token_scores) and commits the sequence.  Results equal the
+// two-kernel path bit for bit.
+template <int VPT>
+__global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dims dm, BandRows rows,
+                                                                 int64_t row_stride,
+                                                                 const int32_t* __restrict__ seq_ids,
+                                                                 const int32_t* __restrict__ cu_new) {
+  const int band = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x;
+  const int seq = seq_ids[b];
+  const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > 1 || cu_new[0] != 0) {
+    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  if (n_new == 0) return;
+  const int nb = dm.nA + dm.nB;
+  const int nc0 = st.n_cache[seq];
+  const int pos = st.n_seen[seq];
+  if (nc0 + 1 > dm.T) {
+    if (tid == 0 && band == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+    return;
+  }
+  __shared__ int s_last;
+  band_token_g<VPT>(st, dm, rows, row_stride, band, seq, r0, pos, st.hp_parity[seq]);
+  if (tid == 0) {
     __threadfence();
     s_last = atomicAdd(&st.ticket[seq], 1u) == (unsigned)(nb - 1);
   }
   __syncthreads();
   if (!s_last) return;
-
-  // ---- the last CTA of the sequence: z of every band, the score, the commit
   __threadfence();
-  extern __shared__ float win[];  // [nb][w]: win[band * w + k] = g at position pos - k
-  const int w = dm.z_window;
-  const int n = pos >= 1 ? min(w, pos) : 0;
-  for (int idx = tid; idx < nb * n; idx += kGThreads) {
-    const int bb = idx / n, k = idx - bb * n;
-    win[bb * w + k] = __ldcg(st.g_ring + ((size_t)seq * nb + bb) * dm.G + ((pos - k) & Gm));
+  extern __shared__ float win[];  // [nb][z_window]
+  band_token_scores(st, dm, seq, nc0, pos, win);
+  if (tid == 0) token_commit(st, dm, seq, nc0, pos);
+}
+
+// One new token per sequence with a K/V kind (and any band kinds): the whole
+// score update in one launch.  grid (band layers + L or 2L, batch entries),
+// kGThreads threads: the first CTAs form the band rows' g (band_token_g), the
+// others the (layer, K|V) streams (lag_stream, the multi-token kernel's own
+// code on a one-token call): a layer's K and V in the two halves of a CTA
+// (`half`, when H*d/8 <= 128), else one stream per CTA; the last CTA of a
+// sequence (ticket) forms every kind's score (band_token_scores,
+// kv_token_scores) and commits.  Results equal the three-kernel path bit for
+// bit.
+template <int LH>
+__global__ void __launch_bounds__(kGThreads, EPIKV_TOKEN_MINB) token_kernel(DevState st, Dims dm, BandRows rows, int64_t row_stride,
+                                                           KvDev kv, const int32_t* __restrict__ seq_ids,
+                                                           const int32_t* __restrict__ cu_new, int vpt, int half) {
+  const int b = blockIdx.y, tid = threadIdx.x;
+  const int seq = seq_ids[b];
+  const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
+  if (seq < 0 || seq >= dm.S || n_new < 0 || n_new > 1 || cu_new[0] != 0) {
+    if (tid == 0 && blockIdx.x == 0) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  if (n_new == 0) return;
+  const int nbc = (dm.kinds & kBandKinds) ? dm.nA + dm.nB : 0;  // band CTAs
+  const int nc0 = st.n_cache[seq];
+  const int pos = st.n_seen[seq];
+  if (nc0 + 1 > dm.T) {
+    if (tid == 0 && blockIdx.x == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
+    return;
+  }
+  __shared__ int s_last;
+  if ((int)blockIdx.x < nbc) {
+    const int par = st.hp_parity[seq];
+    if (vpt == 1) band_token_g<1>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
+    else if (vpt == 2) band_token_g<2>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
+    else band_token_g<4>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
+  } else {
+    const int sidx = blockIdx.x - nbc;
+    const int layer = half ? sidx : sidx >> 1;
+    // the new row's slot: this layer's own length under per-layer budgets
+    const int lnc0 = dm.layer_budgets ? st.n_layer[seq * dm.L + layer] : nc0;
+    if (half) lag_stream<LH, 1, true>(st, dm, kv, seq, 1, layer, threadIdx.x >> 7, lnc0);
+    else lag_stream<LH, 1>(st, dm, kv, seq, 1, layer, sidx & 1, lnc0);
   }
   __syncthreads();
-  if (warp == 0) {
-    const int lpt = nb <= 16 ? 16 : 32;  // the lanes of one token, as in score_finalize_kernel
-    const int bl = lane % lpt;
-    const bool live = lane < lpt && pos >= 1 && bl < nb;
-    float za = 0.f, zb = 0.f, ma = 0.f, mb = 0.f;
-    if (live) {
-      const float* row = win + bl * w;  // row[k] = g at position pos - k
-      if (dm.kinds & EPIKV_SCORE_BANDZ) {
-        const float gnew = row[0];
-        float dsum = 0.f;
-        for (int k = 0; k < n; ++k) dsum += row[k] - gnew;
-        const float mean_d = dsum / (float)n;
-        float dev = 0.f;
-        for (int k = 0; k < n; ++k) {
-          const float e = (row[k] - gnew) - mean_d;
-          dev = fmaf(e, e, dev);
-        }
-        const float sigma = sqrtf(dev / (float)n);
-        const float z = -mean_d / (sigma + dm.z_eps);
-        if (bl < dm.nA) za = z; else zb = z;
-      }
-      if (dm.kinds & EPIKV_SCORE_HSVAR) {
-        float sum = 0.f;
-        for (int k = 0; k < n; ++k) sum += row[k];
-        const float gbar = sum / (float)n;
-        if (bl < dm.nA) ma = gbar; else mb = gbar;
-      }
-    }
-    for (int o = lpt >> 1; o > 0; o >>= 1) {
-      za += __shfl_xor_sync(0xffffffffu, za, o);
-      zb += __shfl_xor_sync(0xffffffffu, zb, o);
-      ma += __shfl_xor_sync(0xffffffffu, ma, o);
-      mb += __shfl_xor_sync(0xffffffffu, mb, o);
-    }
-    if (lane == 0) {
-      const size_t slot = (size_t)seq * dm.T + nc0;
-      st.pos[slot] = pos;
-      if (dm.kinds & EPIKV_SCORE_BANDZ) st.score[0][slot] = pos >= 1 ? za / (float)dm.nA - zb / (float)dm.nB : 0.f;
-      if (dm.kinds & EPIKV_SCORE_HSVAR) st.score[2][slot] = pos >= 1 ? ma / (float)dm.nA - mb / (float)dm.nB : 0.f;
-      if (dm.layer_budgets) {  // the new token is in every layer
-        st.lmask[slot] = dm.L == 64 ? ~0ull : (1ull << dm.L) - 1ull;
-        for (int l = 0; l < dm.L; ++l) {
-          st.n_layer[seq * dm.L + l] += 1;
-          st.lfirst[seq * dm.L + l] = st.n_layer[seq * dm.L + l];
-        }
-      }
-      if (st.first_changed[seq] < nc0) set_error(st.err, EPIKV_DEV_KEPT);  // as in score_finalize_kernel
-      st.first_changed[seq] = nc0 + 1;
-      st.n_cache[seq] = nc0 + 1;
-      st.n_seen[seq] = pos + 1;
-      st.hp_parity[seq] = par ^ 1;
-      atomicAdd(&st.stats[0], 1ull);
-      st.ticket[seq] = 0u;
-    }
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(&st.ticket[seq], 1u) == gridDim.x - 1;
   }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  extern __shared__ float win[];  // [nb][z_window] (band kinds)
+  if (nbc) band_token_scores(st, dm, seq, nc0, pos, win);
+  if (tid < 32) kv_token_scores(st, dm, seq, nc0, pos);
+  if (tid == 0) token_commit(st, dm, seq, nc0, pos);
 }
 
 // ------------------------------------------------------------------ launchers
@@ -772,6 +923,12 @@ cudaError_t finalize_prepare() {
   const int mx = (int)((size_t)kMaxBand * (kFinTile + kMaxWindow - 1) * sizeof(float));
   const int wmx = (int)((size_t)kMaxBand * kMaxWindow * sizeof(float));
   cudaError_t e = cudaFuncSetAttribute(bandz_token_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
   if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
@@ -799,6 +956,28 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
       bandz_token_kernel<2><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
     else
       bandz_token_kernel<4><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
+    ++*launches;
+    return cudaGetLastError();
+  }
+  if (max_new == 1 && dm.L <= 64) {  // a decode step with a K/V kind: one fused launch
+    BandRows rows;
+    const bool band = dm.kinds & kBandKinds;
+    for (int i = 0; i < kMaxBand; ++i)
+      rows.p[i] = band && i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
+    const int vr = dm.D / 8;
+    const int vpt = vr <= kGThreads ? 1 : vr <= 2 * kGThreads ? 2 : 4;
+    const int half = dm.H * dm.d / 8 <= 128;  // a layer's K and V streams share a CTA
+    const dim3 grid((band ? nb : 0) + (half ? dm.L : 2 * dm.L), n_seq);
+    const size_t wsm = band ? (size_t)nb * dm.z_window * sizeof(float) : 0;
+    const int64_t rs = band ? hv->row_stride : 0;
+    switch (dm.d / 8) {
+      case 1: token_kernel<1><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      case 2: token_kernel<2><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      case 4: token_kernel<4><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      case 8: token_kernel<8><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      case 16: token_kernel<16><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      default: token_kernel<32><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+    }
     ++*launches;
     return cudaGetLastError();
   }
