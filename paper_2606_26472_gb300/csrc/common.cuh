@@ -86,6 +86,49 @@ struct KvDev {
   int64_t table_stride_layer;  // elements between layers' block tables (0: shared)
 };
 
+// Programmatic dependent launch.  The kernels of a step are launched with
+// programmatic stream serialisation (pdl_launch): each may be scheduled while
+// the kernel before it on the stream finishes, and waits in pdl_wait -- its
+// first statement -- until that kernel has completed and its writes are
+// visible; pdl_trigger lets the next kernel be scheduled once every CTA of
+// this one has started.  Launched without the attribute, both are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+#ifndef EPIKV_PDL
+#define EPIKV_PDL 1  // 0: plain stream order
+#endif
+
+template <typename... Params, typename... Args>
+inline cudaError_t launch_kernel(bool programmatic, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                                 cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = programmatic && EPIKV_PDL ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+template <typename... Params, typename... Args>
+inline cudaError_t pdl_launch(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              Args... args) {
+  return launch_kernel(true, kernel, grid, block, smem, stream, args...);
+}
+
+// Plain stream order: the long copy kernel, whose CTAs spread more evenly
+// when none of them is placed before the kernel ahead of it has finished.
+template <typename... Params, typename... Args>
+inline cudaError_t plain_launch(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                                Args... args) {
+  return launch_kernel(false, kernel, grid, block, smem, stream, args...);
+}
+
 __device__ __forceinline__ void set_error(int32_t* err, int code) {
   atomicCAS(err, 0, code);
 }

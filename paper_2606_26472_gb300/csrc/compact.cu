@@ -156,6 +156,8 @@ template <bool kLayers>
 __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev kv,
                                                      const int32_t* __restrict__ seq_ids, int n_seq,
                                                      const int32_t* __restrict__ kept, int kept_stride) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ __align__(8) uint64_t full[kStages];
   __shared__ char* dptr[kStages][kMaxRPB];
@@ -414,6 +416,8 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
                                                                       const int32_t* __restrict__ seq_ids,
                                                                       int n_seq, const int32_t* __restrict__ kept,
                                                                       int kept_stride) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ __align__(128) unsigned char smem[];
   int* list = reinterpret_cast<int*>(smem);
   int64_t* pre = reinterpret_cast<int64_t*>(list + list_ints(n_seq));
@@ -482,6 +486,8 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
 
 // The batch entries' evictions have been applied: nothing is left pending.
 __global__ void compact_consumed_kernel(DevState st, Dims dm, const int32_t* __restrict__ seq_ids, int n_seq) {
+  pdl_wait();
+  pdl_trigger();
   for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < n_seq; b += gridDim.x * blockDim.x) {
     const int seq = seq_ids[b];
     if (seq < 0 || seq >= dm.S) continue;
@@ -526,22 +532,23 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
                            cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
   cudaError_t e = cudaSuccess;
+  const size_t smem = compact_smem(n_seq);
   if (dm.layer_budgets) {
-    compact_kernel<true><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+    plain_launch(compact_kernel<true>, ctas, 32, smem, stream, st, dm, kv, seq_ids, n_seq, kept, kept_stride);
   } else {
     if (ctas <= kMaxStashCtas) {  // the balanced split's stash (the kernel checks whether it applies)
-      compact_stash_kernel<<<ctas, kStashThreads, stash_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept,
-                                                                              kept_stride);
+      pdl_launch(compact_stash_kernel, ctas, kStashThreads, stash_smem(n_seq), stream, st, dm, kv, seq_ids, n_seq,
+                 kept, kept_stride);
       ++*launches;
       e = cudaGetLastError();
       if (e != cudaSuccess) return e;
     }
-    compact_kernel<false><<<ctas, 32, compact_smem(n_seq), stream>>>(st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+    plain_launch(compact_kernel<false>, ctas, 32, smem, stream, st, dm, kv, seq_ids, n_seq, kept, kept_stride);
   }
   ++*launches;
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  compact_consumed_kernel<<<(n_seq + 255) / 256, 256, 0, stream>>>(st, dm, seq_ids, n_seq);
+  pdl_launch(compact_consumed_kernel, (n_seq + 255) / 256, 256, 0, stream, st, dm, seq_ids, n_seq);
   ++*launches;
   return cudaGetLastError();
 }

@@ -48,6 +48,8 @@ __global__ void __launch_bounds__(kGThreads, (EPIKV_G_MINB > 0 ? EPIKV_G_MINB : 
                                                             const int32_t* __restrict__ seq_ids,
                                                             const int32_t* __restrict__ cu_new, int n_seq,
                                                             int max_new) {
+  pdl_wait();
+  pdl_trigger();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // the whole batch must be well formed, else nothing is read
   __shared__ int bad;
@@ -448,6 +450,8 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
                                                              const int32_t* __restrict__ seq_ids,
                                                              const int32_t* __restrict__ cu_new,
                                                              int max_new) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y;
   const int seq = seq_ids[b];
   const int n_new = cu_new[b + 1] - cu_new[b];
@@ -478,6 +482,8 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
                                                                      const int32_t* __restrict__ seq_ids,
                                                                      const int32_t* __restrict__ cu_new,
                                                                      int max_new) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y;
   const int seq = seq_ids[b];
   const int n_new = cu_new[b + 1] - cu_new[b];
@@ -826,6 +832,8 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
                                                                  int64_t row_stride,
                                                                  const int32_t* __restrict__ seq_ids,
                                                                  const int32_t* __restrict__ cu_new) {
+  pdl_wait();
+  pdl_trigger();
   const int band = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;
   const int seq = seq_ids[b];
@@ -869,6 +877,8 @@ template <int LH>
 __global__ void __launch_bounds__(kGThreads, EPIKV_TOKEN_MINB) token_kernel(DevState st, Dims dm, BandRows rows, int64_t row_stride,
                                                            KvDev kv, const int32_t* __restrict__ seq_ids,
                                                            const int32_t* __restrict__ cu_new, int vpt, int half) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y, tid = threadIdx.x;
   const int seq = seq_ids[b];
   const int r0 = cu_new[b], n_new = cu_new[b + 1] - r0;
@@ -922,73 +932,71 @@ static size_t finalize_smem(const Dims& dm) {
 cudaError_t finalize_prepare() {
   const int mx = (int)((size_t)kMaxBand * (kFinTile + kMaxWindow - 1) * sizeof(float));
   const int wmx = (int)((size_t)kMaxBand * kMaxWindow * sizeof(float));
-  cudaError_t e = cudaFuncSetAttribute(bandz_token_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(token_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(bandz_token_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, wmx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(score_finalize_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  cudaError_t e = cudaSuccess;
+  auto allow = [&](auto kern, int bytes) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  };
+  allow(bandz_token_kernel<1>, wmx);
+  allow(bandz_token_kernel<2>, wmx);
+  allow(bandz_token_kernel<4>, wmx);
+  allow(token_kernel<1>, wmx);
+  allow(token_kernel<2>, wmx);
+  allow(token_kernel<4>, wmx);
+  allow(token_kernel<8>, wmx);
+  allow(token_kernel<16>, wmx);
+  allow(token_kernel<32>, wmx);
+  allow(score_finalize_kernel<1>, mx);
+  allow(score_finalize_kernel<2>, mx);
+  allow(score_finalize_kernel<4>, mx);
+  allow(score_finalize_kernel<8>, mx);
+  allow(score_finalize_kernel<32>, mx);
   return e;
 }
+
 cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, const int32_t* seq_ids,
                                 const int32_t* cu_new, int max_new, const epikv_hidden_view* hv,
                                 const KvDev* kv, int num_sms, cudaStream_t stream, int* launches) {
   if (n_seq == 0 || max_new == 0) return cudaSuccess;
   const int nb = dm.nA + dm.nB;
+  const bool band = dm.kinds & kBandKinds;
+  BandRows rows;
+  for (int i = 0; i < kMaxBand; ++i)
+    rows.p[i] = band && i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
+  const int64_t rs = band ? hv->row_stride : 0;
+  const int vr = dm.D / 8;
+  const int vpt = vr <= kGThreads ? 1 : vr <= 2 * kGThreads ? 2 : 4;  // band row vectors per thread
   if (max_new == 1 && !(dm.kinds & kKvKinds)) {  // a decode step of the band kinds: one fused launch
-    BandRows rows;
-    for (int i = 0; i < kMaxBand; ++i)
-      rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
-    const int vr = dm.D / 8;
     const dim3 grid(nb, n_seq);
     const size_t wsm = (size_t)nb * dm.z_window * sizeof(float);  // the last CTA's staged windows
-    if (vr <= kGThreads)
-      bandz_token_kernel<1><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
-    else if (vr <= 2 * kGThreads)
-      bandz_token_kernel<2><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
-    else
-      bandz_token_kernel<4><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new);
+    auto go = [&](auto kern) { pdl_launch(kern, grid, kGThreads, wsm, stream, st, dm, rows, rs, seq_ids, cu_new); };
+    if (vpt == 1) go(bandz_token_kernel<1>);
+    else if (vpt == 2) go(bandz_token_kernel<2>);
+    else go(bandz_token_kernel<4>);
     ++*launches;
     return cudaGetLastError();
   }
   if (max_new == 1 && dm.L <= 64) {  // a decode step with a K/V kind: one fused launch
-    BandRows rows;
-    const bool band = dm.kinds & kBandKinds;
-    for (int i = 0; i < kMaxBand; ++i)
-      rows.p[i] = band && i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
-    const int vr = dm.D / 8;
-    const int vpt = vr <= kGThreads ? 1 : vr <= 2 * kGThreads ? 2 : 4;
     const int half = dm.H * dm.d / 8 <= 128;  // a layer's K and V streams share a CTA
     const dim3 grid((band ? nb : 0) + (half ? dm.L : 2 * dm.L), n_seq);
     const size_t wsm = band ? (size_t)nb * dm.z_window * sizeof(float) : 0;
-    const int64_t rs = band ? hv->row_stride : 0;
+    auto go = [&](auto kern) {
+      pdl_launch(kern, grid, kGThreads, wsm, stream, st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half);
+    };
     switch (dm.d / 8) {
-      case 1: token_kernel<1><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
-      case 2: token_kernel<2><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
-      case 4: token_kernel<4><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
-      case 8: token_kernel<8><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
-      case 16: token_kernel<16><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
-      default: token_kernel<32><<<grid, kGThreads, wsm, stream>>>(st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half); break;
+      case 1: go(token_kernel<1>); break;
+      case 2: go(token_kernel<2>); break;
+      case 4: go(token_kernel<4>); break;
+      case 8: go(token_kernel<8>); break;
+      case 16: go(token_kernel<16>); break;
+      default: go(token_kernel<32>); break;
     }
     ++*launches;
     return cudaGetLastError();
   }
-  if (dm.kinds & kBandKinds) {
-    BandRows rows;
-    for (int i = 0; i < kMaxBand; ++i)
-      rows.p[i] = i < nb ? static_cast<const __nv_bfloat16*>(hv->band_rows[i]) : nullptr;
+  if (band) {
     // persistent: as many CTAs as are resident, never more than rows
     static int resident[3] = {0, 0, 0};
-    const int vr = dm.D / 8;
-    const int vi = vr <= kGThreads ? 0 : vr <= 2 * kGThreads ? 1 : 2;
+    const int vi = vpt == 1 ? 0 : vpt == 2 ? 1 : 2;
     if (!resident[vi]) {
       int per_sm = 1;
       if (vi == 0) cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bandz_g_kernel<1>, kGThreads, 0);
@@ -998,42 +1006,39 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
     }
     const int64_t rows_bound = (int64_t)nb * n_seq * max_new;
     const int grid = (int)(rows_bound < resident[vi] ? rows_bound : resident[vi]);
-    if (vi == 0)
-      bandz_g_kernel<1><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
-    else if (vi == 1)
-      bandz_g_kernel<2><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
-    else
-      bandz_g_kernel<4><<<grid, kGThreads, 0, stream>>>(st, dm, rows, hv->row_stride, seq_ids, cu_new, n_seq, max_new);
+    auto go = [&](auto kern) {
+      pdl_launch(kern, grid, kGThreads, 0, stream, st, dm, rows, rs, seq_ids, cu_new, n_seq, max_new);
+    };
+    if (vi == 0) go(bandz_g_kernel<1>);
+    else if (vi == 1) go(bandz_g_kernel<2>);
+    else go(bandz_g_kernel<4>);
     ++*launches;
   }
   if (dm.kinds & kKvKinds) {
-    dim3 grid(2 * dm.L, n_seq);
+    const dim3 grid(2 * dm.L, n_seq);
     const int threads = max(32, (dm.H * dm.d / 8 + 31) / 32 * 32);
+    auto go = [&](auto kern) { pdl_launch(kern, grid, threads, 0, stream, st, dm, *kv, seq_ids, cu_new, max_new); };
     switch (dm.d / 8) {
-      case 1: lagkv_partial_kernel<1><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
-      case 2: lagkv_partial_kernel<2><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
-      case 4: lagkv_partial_kernel<4><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
-      case 8: lagkv_partial_kernel<8><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
-      case 16: lagkv_partial_kernel<16><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
-      default: lagkv_partial_kernel<32><<<grid, threads, 0, stream>>>(st, dm, *kv, seq_ids, cu_new, max_new); break;
+      case 1: go(lagkv_partial_kernel<1>); break;
+      case 2: go(lagkv_partial_kernel<2>); break;
+      case 4: go(lagkv_partial_kernel<4>); break;
+      case 8: go(lagkv_partial_kernel<8>); break;
+      case 16: go(lagkv_partial_kernel<16>); break;
+      default: go(lagkv_partial_kernel<32>); break;
     }
     ++*launches;
   }
   {
-    dim3 grid((max_new + kFinTile - 1) / kFinTile, n_seq);
-    const int wmax = max((dm.kinds & kBandKinds) ? dm.z_window : 1, (dm.kinds & kKvKinds) ? dm.lag_window : 1);
+    const dim3 grid((max_new + kFinTile - 1) / kFinTile, n_seq);
+    const int wmax = max(band ? dm.z_window : 1, (dm.kinds & kKvKinds) ? dm.lag_window : 1);
     const int wpl = (wmax + 31) / 32;
     const size_t smem = finalize_smem(dm);
-    if (wpl <= 1)
-      score_finalize_kernel<1><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
-    else if (wpl <= 2)
-      score_finalize_kernel<2><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
-    else if (wpl <= 4)
-      score_finalize_kernel<4><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
-    else if (wpl <= 8)
-      score_finalize_kernel<8><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
-    else
-      score_finalize_kernel<32><<<grid, kFinThreads, smem, stream>>>(st, dm, seq_ids, cu_new, max_new);
+    auto go = [&](auto kern) { pdl_launch(kern, grid, kFinThreads, smem, stream, st, dm, seq_ids, cu_new, max_new); };
+    if (wpl <= 1) go(score_finalize_kernel<1>);
+    else if (wpl <= 2) go(score_finalize_kernel<2>);
+    else if (wpl <= 4) go(score_finalize_kernel<4>);
+    else if (wpl <= 8) go(score_finalize_kernel<8>);
+    else go(score_finalize_kernel<32>);
     ++*launches;
   }
   return cudaGetLastError();

@@ -244,6 +244,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
                                                              int32_t* __restrict__ kept_out, int kept_stride,
                                                              int32_t* __restrict__ n_kept_out, int staged_cap,
                                                              int smem_words) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x, tid = threadIdx.x;
   const int seq = seq_ids[b];
   if (seq < 0 || seq >= dm.S) {
@@ -446,6 +448,8 @@ __global__ void __launch_bounds__(kLayerThreads) layer_keep_kernel(DevState st, 
                                                                    const int32_t* __restrict__ trigger,
                                                                    int32_t* __restrict__ kept_out, int kept_stride,
                                                                    int32_t* __restrict__ n_kept_out) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int NT = kLayerThreads, NW = NT / 32;
   const int l = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, L = dm.L;
   const int lane = tid & 31;
@@ -562,6 +566,8 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
                                                                   const int32_t* __restrict__ budget,
                                                                   const int32_t* __restrict__ trigger,
                                                                   int kept_stride, int smem_words) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int NW = kSelThreads / 32;
   const int b = blockIdx.x, tid = threadIdx.x, L = dm.L;
   const int lane = tid & 31;
@@ -654,22 +660,23 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
                           const int32_t* budget, const int32_t* trigger, int32_t* kept, int kept_stride,
                           int32_t* n_kept, cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
+  const size_t smem = sel_smem(dm);
+  const int words = sel_smem_words(dm);
   if (dm.layer_budgets) {
-    layer_keep_kernel<<<dim3(dm.L, n_seq), kLayerThreads, 0, stream>>>(st, dm, seq_ids, budget, trigger, kept,
-                                                                       kept_stride, n_kept);
+    pdl_launch(layer_keep_kernel, dim3(dm.L, n_seq), kLayerThreads, 0, stream, st, dm, seq_ids, budget, trigger,
+               kept, kept_stride, n_kept);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ++*launches;
-    layer_union_kernel<<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept_stride,
-                                                                     sel_smem_words(dm));
-  } else if (dm.select_chunk > 1)
-    select_kernel<true><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
-                                                                      kept_stride, n_kept, sel_staged_cap(dm),
-                                                                      sel_smem_words(dm));
-  else
-    select_kernel<false><<<n_seq, kSelThreads, sel_smem(dm), stream>>>(st, dm, seq_ids, budget, trigger, kept,
-                                                                       kept_stride, n_kept, sel_staged_cap(dm),
-                                                                       sel_smem_words(dm));
+    pdl_launch(layer_union_kernel, n_seq, kSelThreads, smem, stream, st, dm, seq_ids, budget, trigger, kept_stride,
+               words);
+  } else if (dm.select_chunk > 1) {
+    pdl_launch(select_kernel<true>, n_seq, kSelThreads, smem, stream, st, dm, seq_ids, budget, trigger, kept,
+               kept_stride, n_kept, sel_staged_cap(dm), words);
+  } else {
+    pdl_launch(select_kernel<false>, n_seq, kSelThreads, smem, stream, st, dm, seq_ids, budget, trigger, kept,
+               kept_stride, n_kept, sel_staged_cap(dm), words);
+  }
   ++*launches;
   return cudaGetLastError();
 }
