@@ -1029,8 +1029,9 @@ def run_window(args):
                          "frac": ach / peak, "peak_source": peak_src, "traffic": None,
                          "algorithmic_bytes_per_launch": compact_bytes / n_launch,
                          "timing": "eager calls, phase events"},
-            # g, [Lag-KV partial,] finalize, select, stash, compaction, eviction consumed
-            "gpu_launches": (7 if wl.kinds & E.EPIKV_SCORE_LAGKV else 6) * n_launch,
+            # one-token calls: the fused score kernel, select, stash, compaction, eviction
+            # consumed; longer calls: g, [Lag-KV partial,] finalize and the same four
+            "gpu_launches": (5 if C == 1 else (7 if wl.kinds & E.EPIKV_SCORE_LAGKV else 6)) * n_launch,
             "clocks": clk}
     print(json.dumps(line), flush=True)
 
