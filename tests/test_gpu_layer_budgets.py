@@ -253,16 +253,23 @@ def test_config2_shape_with_pyramid_layer_budgets(gpu_lib):
     sess.close()
 
 
-def test_layer_budgets_one_token_per_call(gpu_lib):
-    """Decode steps of the band kinds take the fused g + z kernel, which must
-    also advance every layer's length and mark the new slot in every layer."""
+@pytest.mark.parametrize("kinds,policies", [
+    (BANDZ | E.EPIKV_SCORE_HSVAR, (BANDZ, E.EPIKV_SCORE_HSVAR)),
+    (BANDZ | LAGKV, (LAGKV, BANDZ)),
+    (LAGKV | E.EPIKV_SCORE_KVKEY, (E.EPIKV_SCORE_KVKEY, LAGKV)),
+], ids=["band_kinds", "band_and_lagkv", "kv_kinds"])
+def test_layer_budgets_one_token_per_call(gpu_lib, kinds, policies):
+    """Decode steps take the one-launch score kernels (band kinds alone: the
+    fused g + z kernel; with a K/V kind: the kernel that also runs every
+    layer's K/V streams), which must also advance every layer's length, put
+    each layer's new row in that layer's own next slot and mark the new slot
+    in every layer."""
     model = W.small_model(67)
     L = model.num_layers
-    kinds = BANDZ | E.EPIKV_SCORE_HSVAR
     budgets = [[60, 40, 50, 30], [45, 45, 20, 70]]
     triggers = [max(k) + 3 for k in budgets]
     sess = Session(model, n_seq=2, kinds=kinds, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=80, max_new=1,
-                   prefill=(2, 0), policies=(BANDZ, E.EPIKV_SCORE_HSVAR), layer_budgets=1, layer_tables=True)
+                   prefill=(2, 0), policies=policies, layer_budgets=1, layer_tables=True)
     refs = [OracleTrace(model, sess.dt.tabs, b, 150, kinds) for b in range(2)]
     replay = [LayerReplay(L, budgets[b], sess.prefill[b], triggers[b]) for b in range(2)]
     for step in range(150):

@@ -117,17 +117,19 @@ def test_decode_parity_small(gpu_lib, name, layout, kinds, prefill, budgets, chu
     sess.close()
 
 
-@pytest.mark.parametrize("kinds", [63, E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR], ids=["all_kinds", "band_kinds"])
+@pytest.mark.parametrize("kinds", [63, E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR, 58],
+                         ids=["all_kinds", "band_kinds", "kv_kinds"])
 def test_chunking_invariance_and_causality(gpu_lib, kinds):
     """Scores are identical, bit for bit, however the trace is split into calls
-    (with the band kinds alone, one token per call takes the fused decode
-    kernel and the longer calls the two-kernel path)."""
+    (one token per call takes the one-launch decode kernels -- band kinds
+    alone the fused g + z kernel, with a K/V kind the kernel that also runs
+    the K/V streams -- and the longer calls the multi-kernel path)."""
     model = W.small_model(77)
     L = 200
     results = []
     for chunk in (1, 7, 64, 200):
         sess = Session(model, n_seq=1, kinds=kinds, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=L,
-                       max_new=chunk, prefill=(0,), policies=(1,))
+                       max_new=chunk, prefill=(0,), policies=(kinds & -kinds,))
         while sess.n_seen[0] < L:
             sess.score_update([(0, min(chunk, L - sess.n_seen[0]))])
         results.append([sess.read(0, k)[1] for k in ALL_KINDS if kinds & k])
