@@ -137,6 +137,7 @@ size_t carve(const Dims& d, DevState* st, char* base) {
   }
   st->work = (uint32_t*)take(2 * 4);
   st->stash = (char*)take((size_t)kMaxStashCtas * d.stash_rows * d.H * d.d * 2);
+  st->stash_row0 = (int32_t*)take((size_t)kMaxStashCtas * 4);
   return align_up(off, 256);
 }
 

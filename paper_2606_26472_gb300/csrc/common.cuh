@@ -63,6 +63,7 @@ struct DevState {
   int32_t* mkept;          // [S][T] the select kernel's kept slots of the largest layer (scratch)
   uint32_t* work;          // [2] the compaction's next unit (per-layer budgets) and finished CTAs (0 between launches)
   char* stash;             // [kMaxStashCtas][stash_rows][H*d] bf16: compaction boundary rows (token budgets)
+  int32_t* stash_row0;     // [kMaxStashCtas] the row whose source is each stash's first row
 };
 
 // The balanced compaction split: at most this many CTAs, each with a stash

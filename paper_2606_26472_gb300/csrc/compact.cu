@@ -24,12 +24,13 @@
 // Balanced split (token budgets): the moved rows of all evicting streams,
 // laid end to end, are cut into one equal chunk per CTA, so one evicting
 // sequence still covers the whole grid and no CTA carries a longer share.
-// A chunk that ends inside a stream at slot a still reads slots a ..
-// kept[a-1], which the next chunk overwrites.  compact_stash_kernel copies
-// those slots aside before the compaction starts, and the chunk reads them
-// there.  Their number is at most the eviction's largest shift
-// kept[n-1] - (n-1); when that exceeds the stash, the per-stream units above
-// are used instead.
+// A chunk that ends inside a stream at slot a still reads, for its last rows,
+// sources in [a, n_new) that later chunks overwrite.  compact_stash_kernel
+// copies those rows aside before the compaction starts, and the chunk reads
+// them there.  They are a suffix of the chunk's rows in that stream, no
+// longer than the chunk nor than the eviction's largest shift
+// kept[n-1] - (n-1); when both bounds exceed the stash, the per-stream units
+// above are used instead.
 //
 // A selection's eviction is compacted once: compact_consumed_kernel, launched
 // after the copy, sets each sequence's first moved slot to its length, so
@@ -111,12 +112,16 @@ __device__ int evicting_entries(const DevState& st, const Dims& dm, const int32_
 }
 
 // Whether the balanced split applies: token budgets, a grid within the
-// stash's CTAs, and every evicting entry's largest shift (that of its last
-// kept slot) within one CTA's stash.
+// stash's CTAs, and a bound on the rows of a chunk whose sources lie in later
+// chunks' regions -- a suffix of the chunk's last stream segment, no longer
+// than the segment (so than the chunk, ceil(total / grid) rows) nor than the
+// largest shift kept[n-1] - (n-1) of any evicting entry -- within one CTA's
+// stash.  total = moved rows of all streams.
 __device__ bool balanced_split(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
                                const int* list, int n_ev, const int32_t* __restrict__ kept, int kept_stride,
-                               int lane) {
+                               int64_t total, int lane) {
   if (!EPIKV_COMPACT_BALANCED || dm.layer_budgets || gridDim.x > kMaxStashCtas) return false;
+  if ((total + gridDim.x - 1) / gridDim.x <= dm.stash_rows) return true;
   bool ok = true;
   for (int e = lane; e < n_ev; e += 32) {
     const int b = list[e];
@@ -148,7 +153,9 @@ struct Cursor {
   int i;      // next row of the unit
   int end;    // row past the last of the unit
   int b, seq, layer, kvk, hg;
-  int stash_at;   // balanced: sources at or past this slot are read from the next chunk's stash
+  int stash_at;   // balanced: sources in [stash_at, n_new) are read from the next chunk's stash
+  int n_new;      // balanced: the sequence's length after the eviction
+  int row0;       // balanced: the row whose source is the stash's first row
   int64_t o_end;  // balanced: row `end` in the balanced row space
 };
 
@@ -170,7 +177,8 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   // ---- the batch entries that evicted (every CTA builds the same list)
   const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, kLayers ? nullptr : pre, lane);
   if (n_ev == 0) return;
-  const bool balanced = !kLayers && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, lane);
+  const bool balanced =
+      !kLayers && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, pre[n_ev] * 2 * dm.L, lane);
 
   // ---- per-stream units only: whole token rows unless too few streams
   // evict to give every CTA one (small TMA copies cost much more per byte
@@ -255,6 +263,8 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
     if (o_stop - o < rest) {                             // the chunk ends inside this stream
       c.end = c.i + (int)(o_stop - o);
       c.stash_at = c.end;
+      c.n_new = st.n_cache[c.seq];
+      c.row0 = st.stash_row0[blockIdx.x + 1];            // written by compact_stash_kernel
     } else {
       c.end = c.i + (int)rest;
       c.stash_at = INT_MAX;
@@ -323,9 +333,10 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
         const int from = pk[j];
         const int64_t dof = slot_offset(c.layer, c.seq, i);
         const char* from_ptr = nullptr;
-        if (from >= c.stash_at) {      // saved before the copy: the next chunk overwrites it
-          if (from - c.stash_at < dm.stash_rows)
-            from_ptr = st.stash + ((size_t)(blockIdx.x + 1) * dm.stash_rows + (from - c.stash_at)) * rb;
+        if (from >= c.stash_at && from < c.n_new) {  // saved before the copy: a later chunk overwrites it
+          const int k = i - c.row0;
+          if (k >= 0 && k < dm.stash_rows)
+            from_ptr = st.stash + ((size_t)(blockIdx.x + 1) * dm.stash_rows + k) * rb;
         } else if (from >= i) {
           const int64_t so = slot_offset(c.layer, c.seq, from);
           if (so >= 0) from_ptr = kvb + (so + c.hg * piece_elems) * 2;
@@ -408,10 +419,11 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   }
 }
 
-// Before a balanced compaction: CTA g saves the slots that the chunk ending
-// where chunk g begins (slot a of its stream) reads from the region chunk g
-// overwrites, slots a .. kept[a-1], into stash g.  Nothing of the cache is
-// written, so every read sees the rows as the selection left them.
+// Before a balanced compaction: where chunk g begins inside a stream (row a),
+// CTA g saves into stash g the sources of the previous chunk's rows there
+// that lie in [a, n_new) -- the region later chunks overwrite -- row by row
+// from the first such row (stash_row0[g]).  Nothing of the cache is written,
+// so every read sees the rows as the selection left them.
 __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState st, Dims dm, KvDev kv,
                                                                       const int32_t* __restrict__ seq_ids,
                                                                       int n_seq, const int32_t* __restrict__ kept,
@@ -424,7 +436,8 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   __shared__ int s_nev, s_bal;
   if (threadIdx.x < 32) {
     const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, pre, threadIdx.x);
-    const bool bal = n_ev > 0 && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, threadIdx.x);
+    const bool bal = n_ev > 0 && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride,
+                                                pre[n_ev] * 2 * dm.L, threadIdx.x);
     if (threadIdx.x == 0) {
       s_nev = n_ev;
       s_bal = bal;
@@ -441,13 +454,24 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   locate_row(pre, n_ev, upe, o, e, q, r);
   if (r == 0) return;  // the chunk begins its stream: no other chunk reads its region
   const int b = list[e], seq = seq_ids[b];
-  const int a = st.first_changed[seq] + (int)r;
-  const int x = __ldg(kept + (size_t)b * kept_stride + a - 1) - a + 1;
-  if (x <= 0) return;
-  if (x > dm.stash_rows) {
-    if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_KEPT);
-    return;
-  }
+  const int fe = st.first_changed[seq], n_new = st.n_cache[seq];
+  const int a = fe + (int)r;
+  const int32_t* kl = kept + (size_t)b * kept_stride;
+  // the previous chunk's rows in this stream start at seg_start; those whose
+  // sources lie in [a, n_new) are a suffix [i0, i1) of them, at most
+  // stash_rows long (balanced_split), so inside [lo, a)
+  const int64_t s0 = pre[e] * upe + (int64_t)q * (pre[e + 1] - pre[e]);
+  const int64_t o_prev = (int64_t)(blockIdx.x - 1) * total / gridDim.x;
+  const int seg_start = fe + (int)(o_prev > s0 ? o_prev - s0 : 0);
+  const int lo = max(seg_start, a - dm.stash_rows);
+  const int t = threadIdx.x;
+  __shared__ int s_src[kStashRows];  // the sources of rows lo .. a-1
+  const int src = t < a - lo ? __ldg(kl + lo + t) : INT_MAX;
+  if (t < a - lo) s_src[t] = src;
+  const int i0 = lo + __syncthreads_count(src < a);      // kept is increasing: counts of prefixes
+  const int i1 = lo + __syncthreads_count(src < n_new);
+  if (t == 0) st.stash_row0[blockIdx.x] = i0;
+  const int x = i1 - i0;
   const int layer = q >> 1;
   const char* kvb = (q & 1) ? kv.base[1] : kv.base[0];
   const int v16 = dm.H * dm.d / 8;  // 16-byte vectors per row
@@ -457,27 +481,27 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   for (int r0 = warp; r0 < x; r0 += 2 * kWarps) {
     const int r1 = r0 + kWarps;
-    const int64_t s0 = kv_row_offset(kv, layer, seq, a + r0, dm.T);
-    const int64_t s1 = r1 < x ? kv_row_offset(kv, layer, seq, a + r1, dm.T) : -2;
-    if ((s0 == -1 || s1 == -1) && lane == 0) set_error(st.err, EPIKV_DEV_SLOT);
-    const uint4* p0 = reinterpret_cast<const uint4*>(kvb + s0 * 2);
-    const uint4* p1 = reinterpret_cast<const uint4*>(kvb + s1 * 2);
+    const int64_t f0 = kv_row_offset(kv, layer, seq, s_src[i0 - lo + r0], dm.T);
+    const int64_t f1 = r1 < x ? kv_row_offset(kv, layer, seq, s_src[i0 - lo + r1], dm.T) : -2;
+    if ((f0 == -1 || f1 == -1) && lane == 0) set_error(st.err, EPIKV_DEV_SLOT);
+    const uint4* p0 = reinterpret_cast<const uint4*>(kvb + f0 * 2);
+    const uint4* p1 = reinterpret_cast<const uint4*>(kvb + f1 * 2);
     for (int k0 = lane; k0 < v16; k0 += kStashUnroll * 32) {
       uint4 v0[kStashUnroll], v1[kStashUnroll];
 #pragma unroll
       for (int u = 0; u < kStashUnroll; ++u) {
         const int k = k0 + 32 * u;
         if (k < v16) {
-          if (s0 >= 0) v0[u] = __ldg(p0 + k);
-          if (s1 >= 0) v1[u] = __ldg(p1 + k);
+          if (f0 >= 0) v0[u] = __ldg(p0 + k);
+          if (f1 >= 0) v1[u] = __ldg(p1 + k);
         }
       }
 #pragma unroll
       for (int u = 0; u < kStashUnroll; ++u) {
         const int k = k0 + 32 * u;
         if (k < v16) {
-          if (s0 >= 0) dst[(size_t)r0 * v16 + k] = v0[u];
-          if (s1 >= 0) dst[(size_t)r1 * v16 + k] = v1[u];
+          if (f0 >= 0) dst[(size_t)r0 * v16 + k] = v0[u];
+          if (f1 >= 0) dst[(size_t)r1 * v16 + k] = v1[u];
         }
       }
     }

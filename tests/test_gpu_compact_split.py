@@ -1,12 +1,14 @@
 """The compaction's two work splits on the GPU.
 
-When every evicting entry's largest shift (its last kept slot minus its new
-length minus one) fits the 128-row stash, the moved rows of all streams are
-cut into one equal chunk per CTA and the slots a chunk's left neighbour still
-reads are copied aside first; otherwise each (entry, layer, K|V) stream is one
-unit.  Both must leave every kept row in its slot, byte for byte: these cases
-sit on either side of the bound, give far fewer rows than CTAs, hold fewer
-slots than the stash, and mix entries of both kinds in one batch."""
+The moved rows of all streams are cut into one equal chunk per CTA, the
+sources a chunk still reads from later chunks' regions copied aside first,
+when those rows fit the 128-row stash: when every evicting entry's largest
+shift (its last kept slot minus its new length minus one) is at most 128, or
+when no chunk is longer than 128 rows (ceil(total moved rows / 304 CTAs));
+otherwise each (entry, layer, K|V) stream is one unit.  Both must leave every
+kept row in its slot, byte for byte: these cases reach the split through
+either bound or neither, give far fewer rows than CTAs, hold fewer slots than
+the stash, and mix entries of both kinds in one batch."""
 import numpy as np
 import pytest
 import torch
@@ -64,8 +66,8 @@ def _evict_and_check(sess, budgets, generator_check=True, sampled=0):
 @pytest.mark.parametrize("evict", [1, 128, 129, 300])
 def test_one_full_size_sequence_either_side_of_the_stash_bound(gpu_lib, layout, evict):
     """One 32-layer sequence of 600 tokens cut by `evict` slots: its largest
-    shift is `evict`, so 128 and fewer take the balanced split and 129 and
-    more the per-stream units."""
+    shift is `evict`, within the stash up to 128; above it the chunks (at
+    most 64 x 600 / 304 < 128 rows) are the bound that admits the split."""
     model = gen.TraceModel(0xC0A1 + evict)
     sess = Session(model, n_seq=1, kinds=E.EPIKV_SCORE_LAGKV, layout=layout, max_tokens=640, max_new=200,
                    prefill=(0,), policies=(E.EPIKV_SCORE_LAGKV,))
@@ -104,7 +106,7 @@ def test_cache_smaller_than_the_stash(gpu_lib, layout):
 def test_batch_of_mixed_entries(gpu_lib, big):
     """Seven entries with different first moved slots and lengths, one of
     them untouched; with `big`, one entry's shift (200) exceeds the stash and
-    the whole batch takes the per-stream units."""
+    the short chunks (fewer than 8 x 1,800 / 304 rows) admit the split."""
     n = 7
     sess = Session(W.small_model(0xC0A4 + big), n_seq=n, kinds=E.EPIKV_SCORE_LAGKV, layout=E.EPIKV_LAYOUT_PAGED,
                    max_tokens=512, max_new=256, prefill=(0, 17, 0, 64, 0, 5, 0),
@@ -146,4 +148,23 @@ def test_split_over_repeated_decode_evictions(gpu_lib):
                 events += 1
     assert events >= 8
     assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
+@pytest.mark.parametrize("evict", [100, 300])
+def test_full_size_batch_past_both_bounds(gpu_lib, evict):
+    """Three 32-layer sequences of 1,200 tokens cut by `evict` slots: about
+    3 x 64 x 900 moved rows make chunks of ~570 rows, so a shift of 300
+    leaves the balanced split for the per-stream units, and 100 keeps it."""
+    n = 3
+    model = gen.TraceModel(0xC0A6 + evict)
+    sess = Session(model, n_seq=n, kinds=E.EPIKV_SCORE_LAGKV, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=1216,
+                   max_new=400, prefill=(0,) * n, policies=(E.EPIKV_SCORE_LAGKV,) * n)
+    for _ in range(3):
+        sess.score_update([(b, 400) for b in range(n)])
+    kept = _evict_and_check(sess, [1200 - evict] * n, generator_check=False, sampled=24)
+    shifts = [int(kept[b][-1]) - (len(kept[b]) - 1) for b in range(n)]
+    moved = sum(len(kept[b]) - next(i for i, k in enumerate(kept[b]) if k != i) for b in range(n))
+    assert max(shifts) == evict
+    assert -(-moved * 64 // 304) > 128
     sess.close()
