@@ -821,7 +821,9 @@ def run_layers32k(args):
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src, "traffic": None,
                      "algorithmic_bytes_per_launch": compact_bytes / args.steps},
-        "gpu_launches": 6 * args.steps,   # Lag-KV partial, finalize, layer keep, layer union, compaction, consumed
+        # Lag-KV partial, finalize, layer keep, layer union, [stash: at most 256 (sequence, layer)
+        # pairs,] compaction, consumed
+        "gpu_launches": (7 if Bn * L <= 256 else 6) * args.steps,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

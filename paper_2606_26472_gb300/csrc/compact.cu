@@ -16,10 +16,11 @@
 //
 // Under per-layer budgets (kLayers) each (sequence, layer) has its own kept
 // list, first moved slot and length; the streams and the copy are unchanged.
-// The streams then differ in length (a layer's rows follow its budget), so
-// the CTAs take units from a shared counter instead of a fixed stride, in
-// layer-major order: with budgets that fall with depth, larger streams come
-// first and the greedy assignment ends nearly level.
+// The balanced split then runs over (sequence, layer) pairs of two streams
+// each.  Without it the streams differ in length (a layer's rows follow its
+// budget), so the CTAs take units from a shared counter instead of a fixed
+// stride, in layer-major order: with budgets that fall with depth, larger
+// streams come first and the greedy assignment ends nearly level.
 //
 // Balanced split (token budgets): the moved rows of all evicting streams,
 // laid end to end, are cut into one equal chunk per CTA, so one evicting
@@ -73,8 +74,23 @@ constexpr int kStagedBlocks = EPIKV_COMPACT_STAGED_BLOCKS;
 constexpr int kStashThreads = 512;
 constexpr int kStashUnroll = 4;
 
+// The balanced split's row space is made of pairs: under token budgets one
+// per evicting entry, with its 2L streams; under per-layer budgets one per
+// (evicting entry, layer), with that layer's K and V streams, at most
+// kMaxLayerPairs of them (more: per-stream units).
+// Per-layer budgets, 32 layers, 8,192-slot caches evicting 128 slots per
+// step (compaction ms, balanced / per-stream units): 1 sequence 0.35 / 1.09,
+// 2 sequences 0.68 / 1.24, 8 sequences 2.59 / 2.68, 32 sequences 10.18 /
+// 9.95.  So the balanced split takes at most 256 (entry, layer) pairs.
+#ifndef EPIKV_COMPACT_LAYER_PAIRS
+#define EPIKV_COMPACT_LAYER_PAIRS 256
+#endif
+constexpr int kMaxLayerPairs = EPIKV_COMPACT_LAYER_PAIRS;
 __host__ __device__ inline int list_ints(int n_seq) { return (n_seq + 31) / 32 * 32; }
-__host__ __device__ inline int pre_entries(int n_seq) { return (n_seq + 32) / 32 * 32; }
+__host__ __device__ inline int pairs_cap(int n_seq, int L, bool layers) {
+  return layers ? (n_seq * L < kMaxLayerPairs ? n_seq * L : kMaxLayerPairs) : n_seq;
+}
+__host__ __device__ inline int pre_entries(int cap) { return (cap + 32) / 32 * 32; }
 
 // The batch entries that evicted, in batch order, into list; with pre, the
 // prefix sums of their moved rows per stream (pre[k] = rows of entries
@@ -111,22 +127,84 @@ __device__ int evicting_entries(const DevState& st, const Dims& dm, const int32_
   return n_ev;
 }
 
-// Whether the balanced split applies: token budgets, a grid within the
-// stash's CTAs, and a bound on the rows of a chunk whose sources lie in later
-// chunks' regions -- a suffix of the chunk's last stream segment, no longer
-// than the segment (so than the chunk, ceil(total / grid) rows) nor than the
-// largest shift kept[n-1] - (n-1) of any evicting entry -- within one CTA's
-// stash.  total = moved rows of all streams.
+// Per-layer budgets: the prefix sums over the (entry, layer) pairs of their
+// moved rows per stream (pre[k] = rows of the pairs before the k-th, pair k
+// = entry k / L, layer k % L).  One warp; returns the pairs' total.
+__device__ int64_t layer_pairs(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
+                               const int* list, int n_ev, int64_t* pre, int lane) {
+  const int np = n_ev * dm.L;
+  // every pair's rows first (independent loads, several in flight), then the scan
+#pragma unroll 4
+  for (int k = lane; k < np; k += 32) {
+    const int i = seq_ids[list[k / dm.L]] * dm.L + k % dm.L;
+    pre[k + 1] = max(0, st.n_layer[i] - st.lfirst[i]);
+  }
+  __syncwarp();
+  int64_t acc = 0;
+  for (int base = 0; base < np; base += 32) {
+    const int k = base + lane;
+    const int len = k < np ? (int)pre[k + 1] : 0;
+    int incl = len;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (k < np) pre[k + 1] = acc + incl;
+    acc += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  if (lane == 0) pre[0] = 0;
+  __syncwarp();
+  return acc;
+}
+
+// One pair's stream q (token budgets: layer * 2 + K|V; per-layer budgets:
+// K|V): its entry, sequence, layer, first moved row, new length and kept list.
+struct PairAt {
+  int b, seq, layer, kvk, first, n_new;
+  const int32_t* kl;
+};
+__device__ __forceinline__ PairAt pair_at(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
+                                          const int* list, const int32_t* __restrict__ kept, int kept_stride,
+                                          bool layers, int p, int q) {
+  PairAt a;
+  a.b = list[layers ? p / dm.L : p];
+  a.seq = seq_ids[a.b];
+  if (layers) {
+    a.layer = p % dm.L;
+    a.kvk = q;
+    const int i = a.seq * dm.L + a.layer;
+    a.first = st.lfirst[i];
+    a.n_new = st.n_layer[i];
+    a.kl = kept + ((size_t)a.b * dm.L + a.layer) * kept_stride;
+  } else {
+    a.layer = q >> 1;
+    a.kvk = q & 1;
+    a.first = st.first_changed[a.seq];
+    a.n_new = st.n_cache[a.seq];
+    a.kl = kept + (size_t)a.b * kept_stride;
+  }
+  return a;
+}
+
+// Whether the balanced split applies: a grid within the stash's CTAs, under
+// per-layer budgets no more pairs than kMaxLayerPairs, and a bound on the
+// rows of a chunk whose sources lie in later chunks' regions -- a suffix of
+// the chunk's last stream segment, no longer than the segment (so than the
+// chunk, ceil(total / grid) rows) nor than the largest shift
+// kept[n-1] - (n-1) of any pair -- within one CTA's stash.  total = moved
+// rows of all streams.
 __device__ bool balanced_split(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
                                const int* list, int n_ev, const int32_t* __restrict__ kept, int kept_stride,
-                               int64_t total, int lane) {
-  if (!EPIKV_COMPACT_BALANCED || dm.layer_budgets || gridDim.x > kMaxStashCtas) return false;
+                               bool layers, int n_pairs, int64_t total, int lane) {
+  if (!EPIKV_COMPACT_BALANCED || gridDim.x > kMaxStashCtas) return false;
+  if (layers && n_pairs > kMaxLayerPairs) return false;
   if ((total + gridDim.x - 1) / gridDim.x <= dm.stash_rows) return true;
   bool ok = true;
-  for (int e = lane; e < n_ev; e += 32) {
-    const int b = list[e];
-    const int n = st.n_cache[seq_ids[b]];
-    ok = ok && __ldg(kept + (size_t)b * kept_stride + n - 1) - (n - 1) <= dm.stash_rows;
+#pragma unroll 4
+  for (int k = lane; k < n_pairs; k += 32) {
+    const PairAt a = pair_at(st, dm, seq_ids, list, kept, kept_stride, layers, k, 0);
+    if (a.n_new > a.first) ok &= __ldg(a.kl + a.n_new - 1) - (a.n_new - 1) <= dm.stash_rows;
   }
   return __all_sync(0xffffffffu, ok);
 }
@@ -159,7 +237,11 @@ struct Cursor {
   int64_t o_end;  // balanced: row `end` in the balanced row space
 };
 
-template <bool kLayers>
+// kSplit: the balanced split is compiled in (token budgets always; per-layer
+// budgets when the batch has at most kMaxLayerPairs (entry, layer) pairs --
+// the instance for larger batches keeps the per-stream units' code alone,
+// which measured 6 % faster there than with the split's code beside it).
+template <bool kLayers, bool kSplit>
 __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev kv,
                                                      const int32_t* __restrict__ seq_ids, int n_seq,
                                                      const int32_t* __restrict__ kept, int kept_stride) {
@@ -171,14 +253,25 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   __shared__ int stage_rows[kStages];
   int* list = reinterpret_cast<int*>(smem + kStages * kStageBytes);
   int64_t* pre = reinterpret_cast<int64_t*>(list + list_ints(n_seq));
-  int* bt_s = reinterpret_cast<int*>(pre + pre_entries(n_seq));  // the current sequence's block table
+  // the current sequence's block table
+  int* bt_s = reinterpret_cast<int*>(pre + pre_entries(pairs_cap(n_seq, dm.L, kLayers)));
   const int lane = threadIdx.x;
 
   // ---- the batch entries that evicted (every CTA builds the same list)
   const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, kLayers ? nullptr : pre, lane);
   if (n_ev == 0) return;
-  const bool balanced =
-      !kLayers && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, pre[n_ev] * 2 * dm.L, lane);
+  // ---- the balanced split's pairs and their rows
+  const int n_pairs = kLayers ? n_ev * dm.L : n_ev;
+  const int sp = kLayers ? 2 : 2 * dm.L;  // streams per pair
+  int64_t pair_rows = 0;
+  bool balanced = false;
+  if constexpr (kSplit) {
+    if (!kLayers) pair_rows = pre[n_ev];
+    else if (n_pairs <= kMaxLayerPairs) pair_rows = layer_pairs(st, dm, seq_ids, list, n_ev, pre, lane);
+    balanced = (!kLayers || n_pairs <= kMaxLayerPairs) &&
+               balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, kLayers, n_pairs, pair_rows * sp,
+                              lane);
+  }
 
   // ---- per-stream units only: whole token rows unless too few streams
   // evict to give every CTA one (small TMA copies cost much more per byte
@@ -200,7 +293,7 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   // balanced: this CTA's chunk [o_begin, o_stop) of the row space
   int64_t o_begin = 0, o_stop = 0;
   if (balanced) {
-    const int64_t total = pre[n_ev] * upe;
+    const int64_t total = pair_rows * sp;
     o_begin = (int64_t)blockIdx.x * total / G;
     o_stop = (int64_t)(blockIdx.x + 1) * total / G;
   }
@@ -250,20 +343,21 @@ __global__ void __launch_bounds__(32) compact_kernel(DevState st, Dims dm, KvDev
   };
   // balanced: the stream segment holding row o of the chunk
   auto open_at = [&](Cursor& c, int64_t o) {
-    int e, q;
+    int p, q;
     int64_t r;
-    locate_row(pre, n_ev, upe, o, e, q, r);
-    c.b = list[e];
-    c.seq = seq_ids[c.b];
-    c.layer = q >> 1;
-    c.kvk = q & 1;
+    locate_row(pre, n_pairs, sp, o, p, q, r);
+    const PairAt a = pair_at(st, dm, seq_ids, list, kept, kept_stride, kLayers, p, q);
+    c.b = a.b;
+    c.seq = a.seq;
+    c.layer = a.layer;
+    c.kvk = a.kvk;
     c.hg = 0;
-    const int64_t rest = pre[e + 1] - pre[e] - r;       // rows of the stream from o on
-    c.i = st.first_changed[c.seq] + (int)r;
+    const int64_t rest = pre[p + 1] - pre[p] - r;       // rows of the stream from o on
+    c.i = a.first + (int)r;
     if (o_stop - o < rest) {                             // the chunk ends inside this stream
       c.end = c.i + (int)(o_stop - o);
       c.stash_at = c.end;
-      c.n_new = st.n_cache[c.seq];
+      c.n_new = a.n_new;
       c.row0 = st.stash_row0[blockIdx.x + 1];            // written by compact_stash_kernel
     } else {
       c.end = c.i + (int)rest;
@@ -433,34 +527,43 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   extern __shared__ __align__(128) unsigned char smem[];
   int* list = reinterpret_cast<int*>(smem);
   int64_t* pre = reinterpret_cast<int64_t*>(list + list_ints(n_seq));
-  __shared__ int s_nev, s_bal;
+  const bool layers = dm.layer_budgets;
+  const int sp = layers ? 2 : 2 * dm.L;  // streams per pair
+  __shared__ int s_pairs, s_bal;
+  __shared__ int64_t s_rows;
   if (threadIdx.x < 32) {
-    const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, pre, threadIdx.x);
-    const bool bal = n_ev > 0 && balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride,
-                                                pre[n_ev] * 2 * dm.L, threadIdx.x);
+    const int n_ev = evicting_entries(st, dm, seq_ids, n_seq, list, layers ? nullptr : pre, threadIdx.x);
+    const int n_pairs = layers ? n_ev * dm.L : n_ev;
+    int64_t rows = 0;
+    if (!layers) rows = pre[n_ev];
+    else if (n_pairs <= kMaxLayerPairs) rows = layer_pairs(st, dm, seq_ids, list, n_ev, pre, threadIdx.x);
+    const bool bal = n_ev > 0 && (!layers || n_pairs <= kMaxLayerPairs) &&
+                     balanced_split(st, dm, seq_ids, list, n_ev, kept, kept_stride, layers, n_pairs, rows * sp,
+                                    threadIdx.x);
     if (threadIdx.x == 0) {
-      s_nev = n_ev;
+      s_pairs = n_pairs;
+      s_rows = rows;
       s_bal = bal;
     }
   }
   __syncthreads();
   if (!s_bal || blockIdx.x == 0) return;
-  const int n_ev = s_nev, upe = 2 * dm.L;
-  const int64_t total = pre[n_ev] * upe;
+  const int n_pairs = s_pairs;
+  const int64_t total = s_rows * sp;
   const int64_t o = (int64_t)blockIdx.x * total / gridDim.x;
   if (o >= total) return;
-  int e, q;
+  int p, q;
   int64_t r;
-  locate_row(pre, n_ev, upe, o, e, q, r);
+  locate_row(pre, n_pairs, sp, o, p, q, r);
   if (r == 0) return;  // the chunk begins its stream: no other chunk reads its region
-  const int b = list[e], seq = seq_ids[b];
-  const int fe = st.first_changed[seq], n_new = st.n_cache[seq];
+  const PairAt pa = pair_at(st, dm, seq_ids, list, kept, kept_stride, layers, p, q);
+  const int seq = pa.seq, fe = pa.first, n_new = pa.n_new;
   const int a = fe + (int)r;
-  const int32_t* kl = kept + (size_t)b * kept_stride;
+  const int32_t* kl = pa.kl;
   // the previous chunk's rows in this stream start at seg_start; those whose
   // sources lie in [a, n_new) are a suffix [i0, i1) of them, at most
   // stash_rows long (balanced_split), so inside [lo, a)
-  const int64_t s0 = pre[e] * upe + (int64_t)q * (pre[e + 1] - pre[e]);
+  const int64_t s0 = pre[p] * sp + (int64_t)q * (pre[p + 1] - pre[p]);
   const int64_t o_prev = (int64_t)(blockIdx.x - 1) * total / gridDim.x;
   const int seg_start = fe + (int)(o_prev > s0 ? o_prev - s0 : 0);
   const int lo = max(seg_start, a - dm.stash_rows);
@@ -472,8 +575,8 @@ __global__ void __launch_bounds__(kStashThreads) compact_stash_kernel(DevState s
   const int i1 = lo + __syncthreads_count(src < n_new);
   if (t == 0) st.stash_row0[blockIdx.x] = i0;
   const int x = i1 - i0;
-  const int layer = q >> 1;
-  const char* kvb = (q & 1) ? kv.base[1] : kv.base[0];
+  const int layer = pa.layer;
+  const char* kvb = pa.kvk ? kv.base[1] : kv.base[0];
   const int v16 = dm.H * dm.d / 8;  // 16-byte vectors per row
   uint4* dst = reinterpret_cast<uint4*>(st.stash + (size_t)blockIdx.x * dm.stash_rows * dm.H * dm.d * 2);
   // each warp copies two rows at a time, every lane's loads issued before its stores
@@ -523,30 +626,34 @@ __global__ void compact_consumed_kernel(DevState st, Dims dm, const int32_t* __r
 
 static int g_ctas_per_sm = 0;
 
-static size_t stash_smem(int n_seq) {
-  return (size_t)list_ints(n_seq) * sizeof(int) + (size_t)pre_entries(n_seq) * sizeof(int64_t);
+static size_t stash_smem(int n_seq, int L, bool layers) {
+  return (size_t)list_ints(n_seq) * sizeof(int) + (size_t)pre_entries(pairs_cap(n_seq, L, layers)) * sizeof(int64_t);
 }
 
-static size_t compact_smem(int n_seq) {
-  return (size_t)kStages * kStageBytes + stash_smem(n_seq) + (size_t)kStagedBlocks * sizeof(int);
+static size_t compact_smem(int n_seq, int L, bool layers) {
+  return (size_t)kStages * kStageBytes + stash_smem(n_seq, L, layers) + (size_t)kStagedBlocks * sizeof(int);
 }
 
 cudaError_t compact_prepare(int device, int* ctas_per_sm) {
   (void)device;
-  cudaError_t e = cudaFuncSetAttribute(compact_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)compact_smem(4096));
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(compact_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)compact_smem(4096));
+  const int mx = (int)compact_smem(4096, 64, true);  // the largest batch and pair table
+  cudaError_t e = cudaSuccess;
+  auto allow = [&](auto kern) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+  };
+  allow(compact_kernel<false, true>);
+  allow(compact_kernel<true, true>);
+  allow(compact_kernel<true, false>);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(compact_stash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)stash_smem(4096));
+                             (int)stash_smem(4096, 64, true));
   if (e != cudaSuccess) return e;
   int n = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel<false>, 32, compact_smem(64));
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, compact_kernel<false, true>, 32, compact_smem(64, 32, false));
   if (e != cudaSuccess) return e;
   g_ctas_per_sm = n > 0 ? n : 1;
-  if (EPIKV_COMPACT_CTAS_PER_SM > 0 && EPIKV_COMPACT_CTAS_PER_SM < g_ctas_per_sm) g_ctas_per_sm = EPIKV_COMPACT_CTAS_PER_SM;
+  if (EPIKV_COMPACT_CTAS_PER_SM > 0 && EPIKV_COMPACT_CTAS_PER_SM < g_ctas_per_sm)
+    g_ctas_per_sm = EPIKV_COMPACT_CTAS_PER_SM;
   if (ctas_per_sm) *ctas_per_sm = g_ctas_per_sm;
   return cudaSuccess;
 }
@@ -555,22 +662,24 @@ cudaError_t launch_compact(const DevState& st, const Dims& dm, int n_seq, const 
                            const int32_t* kept, int kept_stride, const KvDev& kv, int ctas,
                            cudaStream_t stream, int* launches) {
   if (n_seq == 0) return cudaSuccess;
-  cudaError_t e = cudaSuccess;
-  const size_t smem = compact_smem(n_seq);
-  if (dm.layer_budgets) {
-    plain_launch(compact_kernel<true>, ctas, 32, smem, stream, st, dm, kv, seq_ids, n_seq, kept, kept_stride);
-  } else {
-    if (ctas <= kMaxStashCtas) {  // the balanced split's stash (the kernel checks whether it applies)
-      pdl_launch(compact_stash_kernel, ctas, kStashThreads, stash_smem(n_seq), stream, st, dm, kv, seq_ids, n_seq,
-                 kept, kept_stride);
-      ++*launches;
-      e = cudaGetLastError();
-      if (e != cudaSuccess) return e;
-    }
-    plain_launch(compact_kernel<false>, ctas, 32, smem, stream, st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  const bool layers = dm.layer_budgets;
+  const bool split = !layers || n_seq * dm.L <= kMaxLayerPairs;  // the balanced split may apply
+  const size_t smem = compact_smem(n_seq, dm.L, layers);
+  if (split && ctas <= kMaxStashCtas) {  // the balanced split's stash (the kernel checks whether it applies)
+    pdl_launch(compact_stash_kernel, ctas, kStashThreads, stash_smem(n_seq, dm.L, layers), stream, st, dm, kv,
+               seq_ids, n_seq, kept, kept_stride);
+    ++*launches;
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
   }
+  auto go = [&](auto kern) {
+    plain_launch(kern, ctas, 32, smem, stream, st, dm, kv, seq_ids, n_seq, kept, kept_stride);
+  };
+  if (!layers) go(compact_kernel<false, true>);
+  else if (split) go(compact_kernel<true, true>);
+  else go(compact_kernel<true, false>);
   ++*launches;
-  e = cudaGetLastError();
+  const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   pdl_launch(compact_consumed_kernel, (n_seq + 255) / 256, 256, 0, stream, st, dm, seq_ids, n_seq);
   ++*launches;

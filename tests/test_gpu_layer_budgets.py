@@ -290,3 +290,40 @@ def test_layer_budgets_one_token_per_call(gpu_lib, kinds, policies):
             _check_layer_bytes(sess, b, l, replay[b].caches[l])
     assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()
+
+
+def test_many_sequences_past_the_pair_limit(gpu_lib):
+    """72 sequences x 4 layers = 288 (sequence, layer) pairs: more than the
+    balanced split takes under per-layer budgets (256), so the copy runs on
+    per-stream units from the shared counter; every layer's slots and bytes
+    follow the per-layer replay."""
+    model = W.small_model(0x1A7E)
+    n_seq, L = 72, model.num_layers
+    budgets = [[60 + (b % 5) * 8, 40 + (b % 3) * 10, 50, 30 + (b % 7) * 4] for b in range(n_seq)]
+    slack = 6
+    triggers = [max(k) + slack for k in budgets]
+    T_cap = max(triggers) + 20 + 1
+    sess = Session(model, n_seq=n_seq, kinds=LAGKV, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=T_cap, max_new=20,
+                   prefill=(0,) * n_seq, policies=(LAGKV,) * n_seq, layer_budgets=1, layer_tables=True)
+    replay = [LayerReplay(L, budgets[b], 0, triggers[b]) for b in range(n_seq)]
+    events = 0
+    for step in range(8):
+        entries = [(b, 20 if (b + step) % 4 else 7) for b in range(n_seq)]
+        before = {b: sess.n_cache[b] for b, _ in entries}
+        sess.score_update(entries)
+        for b, n in entries:
+            pos, sc = sess.read(b, LAGKV)
+            replay[b].append(pos[before[b]:before[b] + n], sc[before[b]:before[b] + n])
+        seqs = list(range(n_seq))
+        sess.select(seqs, budgets, triggers)
+        sess.compact(seqs)
+        for b in seqs:
+            events += replay[b].event()
+            for l in range(L):
+                assert list(sess.read_layer(b, l)) == replay[b].caches[l], f"seq {b} layer {l} step {step}"
+    assert events >= 100
+    for b in (0, 17, 41, 71):
+        for l in range(L):
+            _check_layer_bytes(sess, b, l, replay[b].caches[l])
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
