@@ -8,11 +8,13 @@
 // through a ring of shared-memory stages: while batch k is stored, batches
 // k+1 .. k+S-1 are loading.
 //
-// In-place safety without any inter-CTA wait: streams are disjoint bytes, so
-// one CTA owns each; inside a stream kept[i] >= i and rows are processed in
+// In-place safety without any inter-CTA wait: streams are disjoint bytes;
+// inside a CTA's rows of a stream kept[i] >= i and rows are processed in
 // increasing i, so a load (slot kept[i] >= i) never reads a slot that an
 // earlier store has written, and a later store to a slot some earlier batch
-// still had to read is issued only after that batch's loads completed.
+// still had to read is issued only after that batch's loads completed.  With
+// per-stream units one CTA owns each stream; the balanced split below cuts
+// streams between CTAs and covers the reads across a cut with a stash.
 //
 // Under per-layer budgets (kLayers) each (sequence, layer) has its own kept
 // list, first moved slot and length; the streams and the copy are unchanged.
@@ -22,7 +24,7 @@
 // stride, in layer-major order: with budgets that fall with depth, larger
 // streams come first and the greedy assignment ends nearly level.
 //
-// Balanced split (token budgets): the moved rows of all evicting streams,
+// Balanced split: the moved rows of all evicting streams,
 // laid end to end, are cut into one equal chunk per CTA, so one evicting
 // sequence still covers the whole grid and no CTA carries a longer share.
 // A chunk that ends inside a stream at slot a still reads, for its last rows,
