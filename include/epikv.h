@@ -34,6 +34,13 @@
  *   - bf16 data; K/V rows of one token and layer are H*d contiguous
  *     elements (head-major, channel-minor); all pointers 16-byte aligned.
  *   - A sequence id appears at most once in one call's batch.
+ *   - A call's kernels are launched with programmatic dependent launch
+ *     among themselves (each waits for its predecessor's results before it
+ *     reads anything); against the caller's own work on the stream the
+ *     order is plain stream order, except that a caller kernel itself
+ *     launched with programmatic dependent launch right after a call must,
+ *     as with any such launch, wait for its predecessor
+ *     (cudaGridDependencySynchronize) before reading the call's results.
  */
 #ifndef EPIKV_H_
 #define EPIKV_H_
@@ -169,7 +176,11 @@ typedef struct {
 
 typedef struct epikv_ctx epikv_ctx;
 
-/* Bytes of device workspace epikv_init needs for cfg (0 if cfg is invalid). */
+/* Bytes of device workspace epikv_init needs for cfg (0 if cfg is invalid):
+ * the per-sequence state (counters, frozen scores and positions per slot,
+ * score rings, Lag-KV chunk ranges, kept lists) plus a fixed compaction stash
+ * of 512 x min(128, max_cache_tokens) K/V rows of one layer (128 MiB at
+ * num_kv_heads * head_dim = 1024). */
 size_t epikv_workspace_bytes(const epikv_config* cfg);
 
 /* Create a context over a caller-allocated device workspace of at least
