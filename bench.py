@@ -125,6 +125,7 @@ class Clocks:
     @staticmethod
     def device_id(dev, local_rank):
         """nvidia-smi's --id for torch device `dev`: its UUID, else the local rank."""
+        import torch
         try:
             uuid = str(torch.cuda.get_device_properties(dev).uuid)
             return uuid if uuid.startswith("GPU-") else "GPU-" + uuid
@@ -829,6 +830,29 @@ def run_layers32k(args):
     print(json.dumps(line), flush=True)
 
 
+def window_schedule(n0, budgets, slack, C, n_calls):
+    """The decode window's rows, simulated on the host: per call, every
+    sequence's C new tokens (positions continuing from n0, slots from its
+    cache length), and the sequences that evict (cache length > K + slack,
+    cut back to K).  Returns (positions [n_calls][B*C], slots [n_calls][B*C],
+    evictions per call, cache lengths after the last call)."""
+    B = len(n0)
+    n_cache = np.array(n0, dtype=np.int64)
+    budgets = np.asarray(budgets, dtype=np.int64)
+    pos_tab = np.empty((n_calls, B * C), np.int32)
+    slot_tab = np.empty((n_calls, B * C), np.int32)
+    evict_tab = np.zeros(n_calls, np.int64)
+    r = np.arange(C)
+    for j in range(n_calls):
+        pos_tab[j] = (np.asarray(n0)[:, None] + j * C + r[None, :]).reshape(-1)
+        slot_tab[j] = (n_cache[:, None] + r[None, :]).reshape(-1)
+        n_cache += C
+        ev = n_cache > budgets + slack
+        evict_tab[j] = int(ev.sum())
+        n_cache[ev] = budgets[ev]
+    return pos_tab, slot_tab, evict_tab, n_cache
+
+
 def run_window(args):
     """Steady-state decode windows of two more workloads, timed per
     epikv_step call with CUDA events on the stream; the generator kernels
@@ -911,19 +935,7 @@ def run_window(args):
             dt.kv(b, p0, c, p0, cache.k, cache.v, **cache.synth_kwargs())
             E.epikv_score_update(ctx, 1, ids, cu_s[c], c, hv_s, kv)
 
-    # each call's rows: (sequence, position, slot), simulated on the host
-    n_cache = n0.copy()
-    pos_tab = np.empty((n_calls, Bn * C), np.int32)
-    slot_tab = np.empty((n_calls, Bn * C), np.int32)
-    evict_tab = np.zeros(n_calls, np.int64)
-    r = np.arange(C)
-    for j in range(n_calls):
-        pos_tab[j] = (n0[:, None] + j * C + r[None, :]).reshape(-1)
-        slot_tab[j] = (n_cache[:, None] + r[None, :]).reshape(-1)
-        n_cache += C
-        ev = n_cache > budgets + slack
-        evict_tab[j] = int(ev.sum())
-        n_cache[ev] = budgets[ev]
+    pos_tab, slot_tab, evict_tab, n_cache = window_schedule(n0, budgets, slack, C, n_calls)
     seq_rows = torch.from_numpy(np.repeat(np.arange(Bn, dtype=np.int32), C)).to(dev)
     pos_dev = torch.from_numpy(pos_tab).to(dev)
     slot_dev = torch.from_numpy(slot_tab).to(dev)
