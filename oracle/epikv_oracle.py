@@ -41,8 +41,7 @@ R18 chunk-level selection (named as future work in Sec. 5, after ChunkKV's
     contiguous chunks of Sec. 2): positions fall into fixed chunks
     floor(pos / C); a chunk's score is the mean of the frozen scores of its
     members that are candidates (prefill and recency slots are not members),
-    summed left to right in float32 and divided by the member count in
-    float32, the precision the ranking is decided in on both sides; chunks
+    here in float64 (a correctly rounded sum divided by the count); chunks
     rank by that score (R8's order: NaN lowest, -0 == +0, ties to the
     earlier chunk) and fill the M candidate places whole, in rank order; the
     first chunk that does not fit gives its lowest slots.  C = 1 is R7/R8.
@@ -55,6 +54,8 @@ R19 per-layer budgets (named as future work in Sec. 5, after PyramidKV's
     more than the trigger and more than K_min.  Equal budgets give R7.
 """
 from __future__ import annotations
+
+import math
 
 import numpy as np
 
@@ -247,25 +248,29 @@ def select_kept(scores, K, prefill=0, recency_cap=128):
     return sorted(kept)
 
 
-def chunk_scores(scores, positions, candidates, chunk):
-    """Float32 mean score of every chunk of candidate slots (R18).
+def chunk_mean(values):
+    """Mean of a chunk's member scores (R18): float64, the sum correctly
+    rounded (NaN if any member is NaN)."""
+    values = [float(v) for v in values]
+    if any(math.isnan(v) for v in values):
+        return float("nan")
+    return math.fsum(values) / len(values)
+
+
+def chunk_scores(scores, positions, candidates, chunk, mean=chunk_mean):
+    """Mean score of every chunk of candidate slots (R18).
 
     Returns {chunk id: (mean, [member slots in slot order])}; chunk id =
-    floor(position / chunk).
+    floor(position / chunk).  ``mean`` maps the members' scores (in slot
+    order) to the chunk's score.
     """
     members = {}
     for i in candidates:
         members.setdefault(int(positions[i]) // chunk, []).append(i)
-    out = {}
-    for c, slots in members.items():
-        s = np.float32(0.0)
-        for i in slots:                                   # left to right
-            s = np.float32(s + np.float32(scores[i]))
-        out[c] = (np.float32(s / np.float32(len(slots))), slots)
-    return out
+    return {c: (mean([scores[i] for i in slots]), slots) for c, slots in members.items()}
 
 
-def select_kept_chunked(scores, positions, K, prefill=0, recency_cap=128, chunk=1):
+def select_kept_chunked(scores, positions, K, prefill=0, recency_cap=128, chunk=1, mean=chunk_mean):
     """Ascending kept slot list under chunk-level selection (R18).
 
     Same protected set and budget split as ``select_kept``; the M candidate
@@ -280,7 +285,7 @@ def select_kept_chunked(scores, positions, K, prefill=0, recency_cap=128, chunk=
     R = min(recency_window(K, recency_cap), max(0, K - P))
     M = max(0, K - P - R)
     candidates = list(range(P, n - R))
-    chunks = chunk_scores(scores, positions, candidates, chunk)
+    chunks = chunk_scores(scores, positions, candidates, chunk, mean)
 
     def rank(c):  # NaN last, higher mean first, earlier chunk first
         s = float(chunks[c][0])

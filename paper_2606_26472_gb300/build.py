@@ -1,6 +1,7 @@
 """In-tree build of libepikv.so (and of the synthetic-input generator's
 libepikv_synth.so) for sm_103a with nvcc: one object per translation unit,
-compiled in parallel, linked against the shared CUDA runtime."""
+compiled in parallel, linked against the shared CUDA runtime.  The input
+generator's host twin (libepikv_synth_host.so, plain C) is built with gcc."""
 from __future__ import annotations
 
 import concurrent.futures as cf
@@ -16,6 +17,10 @@ INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libepikv.so")
 SYNTH_DIR = os.path.join(ROOT, "synth")
 SYNTH_LIB = os.path.join(SYNTH_DIR, "libepikv_synth.so")
+SYNTH_HOST_LIB = os.path.join(SYNTH_DIR, "libepikv_synth_host.so")
+# the host twin of the input generator: plain C, every float operation rounded
+# on its own (no contraction), the same bytes on x86-64 and aarch64
+HOST_CFLAGS = ["-O2", "-std=c99", "-fPIC", "-shared", "-ffp-contract=off", "-fno-fast-math"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
@@ -78,6 +83,13 @@ def build(verbose=False):
     _build_so(LIB, srcs, hdrs, [INCLUDE, CSRC], os.path.join(ROOT, "_build", "epikv"), verbose)
     ssrc = [os.path.join(SYNTH_DIR, "synth_gen.cu")]
     _build_so(SYNTH_LIB, ssrc, [], [], os.path.join(ROOT, "_build", "synth"), verbose)
+    hsrc = os.path.join(SYNTH_DIR, "synth_host.c")
+    if _stale(SYNTH_HOST_LIB, [hsrc]):
+        cc = shutil.which("gcc") or shutil.which("cc")
+        if cc is None:
+            raise RuntimeError("no C compiler found for the host input generator")
+        _run([cc, *HOST_CFLAGS, "-o", SYNTH_HOST_LIB + ".tmp", hsrc])
+        os.replace(SYNTH_HOST_LIB + ".tmp", SYNTH_HOST_LIB)
     return LIB
 
 

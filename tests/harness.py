@@ -25,7 +25,7 @@ import torch
 from oracle import epikv_oracle as O
 from paper_2606_26472_gb300 import epikv as E
 from paper_2606_26472_gb300.cache import KVCache
-from synth import gen
+from synth import gen, host
 from synth.device import DeviceTrace, as_u16
 
 TOL = 1e-4
@@ -79,35 +79,100 @@ def assert_scores_close(gpu, ref, what="", cond=None):
         raise AssertionError(f"{what}: {bad.size} scores out of tolerance, first at {i}: gpu {gpu[i]!r} ref {ref[i]!r}")
 
 
+ROW_BLOCK = 2048      # positions generated at a time by the oracle's traces (bounds host memory)
+
+
+def band_g_trace(model, tabs, seq, layer, length, seg):
+    """g_l(t) of one band layer for t < length (g[0] is NaN), Eq. 1: the
+    oracle's hidden_change_trace over blocks of the generator's rows (each
+    block starts one row early so that its first g has its predecessor)."""
+    g = np.full(length, np.nan)
+    for a in range(0, length, ROW_BLOCK):
+        lo, b = max(0, a - 1), min(length, a + ROW_BLOCK)
+        rows = gen.bf16_bits_to_f64(host.hidden_rows(model, tabs, seq, layer, np.arange(lo, b), seg))
+        g[lo + 1:b] = O.hidden_change_trace(rows)[1:]
+    return g
+
+
+def kv_u_traces(model, tabs, seq, length, kinds, lag):
+    """Per-position inputs of the K/V scores' rolling means (Sec. 3.3, R10,
+    R12, R13): {kind: u[0..length)}, each u(t) from the oracle's per-token
+    functions on the generator's rows of t and of its previous lag chunk,
+    generated a block of positions at a time."""
+    sp = gen.spike_flags(model, seq, length)
+    u = {k: np.zeros(length) for k in ALL_KINDS if kinds & k & KV_KINDS}
+    for a in range(0, length, ROW_BLOCK):
+        b = min(length, a + ROW_BLOCK)
+        first = max(0, (a // lag - 1) * lag)            # the previous chunk of a's chunk
+        pos = np.arange(first, b)
+        K = gen.bf16_bits_to_f64(host.kv_rows(model, tabs, seq, 0, pos, sp))
+        V = gen.bf16_bits_to_f64(host.kv_rows(model, tabs, seq, 1, pos, sp))
+        for t in range(a, b):
+            i, c = t - first, t // lag
+            lo = (c - 1) * lag - first
+            if E.EPIKV_SCORE_KVKEY in u:
+                u[E.EPIKV_SCORE_KVKEY][t] = O.head_variance(K[i])
+            if E.EPIKV_SCORE_KVVAL in u:
+                u[E.EPIKV_SCORE_KVVAL][t] = O.head_variance(V[i])
+            if c == 0:
+                continue                                   # u = 0 in chunk 0 (R10)
+            if E.EPIKV_SCORE_LAGKV in u:
+                u[E.EPIKV_SCORE_LAGKV][t] = O.lag_token_variance(K[i], V[i], K[lo:lo + lag], V[lo:lo + lag])
+            if E.EPIKV_SCORE_LAGKEY in u:
+                u[E.EPIKV_SCORE_LAGKEY][t] = O.lag_key_token_variance(K[i], K[lo:lo + lag])
+    return u
+
+
+class _LazyCond:
+    """{kind: kappa[0..length)} of the band-z score, computed on first use."""
+
+    def __init__(self, trace):
+        self._t = trace
+        self._v = None
+
+    def _value(self):
+        if self._v is None:
+            t = self._t
+            self._v = bandz_condition_g(t.g_a, t.g_b, t.z_window)
+        return self._v
+
+    def get(self, kind, default=None):
+        return self._value() if kind == E.EPIKV_SCORE_BANDZ and self._t.has_bandz else default
+
+    def __getitem__(self, kind):
+        v = self.get(kind)
+        if v is None:
+            raise KeyError(kind)
+        return v
+
+
 class OracleTrace:
-    """fp64 oracle scores of one sequence, from the numpy generator's rows."""
+    """fp64 oracle scores of one sequence, positions 0..length-1, from the
+    generator's rows (regenerated block by block by the host twin).
+
+    Band kinds: every band layer's g trace (Eq. 1), then the oracle's rolling
+    z-score and band combination (Eq. 3) or rolling band mean (Eq. 2).  K/V
+    kinds: u(t) per position (Sec. 3.3), then the oracle's rolling mean."""
 
     def __init__(self, model, tabs, seq, length, kinds, z_window=64, lag=16, lag_window=64):
         self.length = length
-        pos = np.arange(length)
+        self.z_window = z_window
         self.scores = {}
-        self.cond = {}    # per-position sensitivity of a kind's score to fp32 rounding of its inputs
-        if kinds & (E.EPIKV_SCORE_BANDZ | E.EPIKV_SCORE_HSVAR):
+        self.has_bandz = bool(kinds & E.EPIKV_SCORE_BANDZ)
+        self.cond = _LazyCond(self)   # per-position sensitivity of the band-z score to fp32 rounding of g
+        if kinds & BAND_KINDS:
             seg = gen.segment_index(model, seq, length)
-            ra = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_a]
-            rb = [gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg)) for l in model.band_b]
+            self.g_a = [band_g_trace(model, tabs, seq, l, length, seg) for l in model.band_a]
+            self.g_b = [band_g_trace(model, tabs, seq, l, length, seg) for l in model.band_b]
             if kinds & E.EPIKV_SCORE_BANDZ:
-                self.scores[E.EPIKV_SCORE_BANDZ] = O.bandz_scores(ra, rb, z_window)
-                self.cond[E.EPIKV_SCORE_BANDZ] = bandz_condition(ra, rb, z_window)
+                self.scores[E.EPIKV_SCORE_BANDZ] = O.epiphany_score(
+                    [O.rolling_zscore(g, z_window) for g in self.g_a], [O.rolling_zscore(g, z_window) for g in self.g_b])
             if kinds & E.EPIKV_SCORE_HSVAR:
-                self.scores[E.EPIKV_SCORE_HSVAR] = O.hsvar_scores(ra, rb, z_window)
+                self.scores[E.EPIKV_SCORE_HSVAR] = (np.mean([O.rolling_band_mean(g, z_window) for g in self.g_a], axis=0)
+                                                    - np.mean([O.rolling_band_mean(g, z_window) for g in self.g_b], axis=0))
         if kinds & KV_KINDS:
-            sp = gen.spike_flags(model, seq, length)
-            K = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0, pos, sp))
-            V = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 1, pos, sp))
-            if kinds & E.EPIKV_SCORE_LAGKV:
-                self.scores[E.EPIKV_SCORE_LAGKV] = O.lagkv_scores(K, V, lag, w=lag_window)
-            if kinds & E.EPIKV_SCORE_LAGKEY:
-                self.scores[E.EPIKV_SCORE_LAGKEY] = O.lag_key_scores(K, lag, w=lag_window)
-            if kinds & E.EPIKV_SCORE_KVKEY:
-                self.scores[E.EPIKV_SCORE_KVKEY] = O.kv_variance_scores(K, lag_window)
-            if kinds & E.EPIKV_SCORE_KVVAL:
-                self.scores[E.EPIKV_SCORE_KVVAL] = O.kv_variance_scores(V, lag_window)
+            for kind, u in kv_u_traces(model, tabs, seq, length, kinds, lag).items():
+                self.scores[kind] = O.rolling_mean(u, lag_window)
 
 
 def _trace_check(self, kind, pos, gpu, what=""):
@@ -291,10 +356,24 @@ class Session:
         E.epikv_destroy(self.ctx)
 
 
+def kernel_chunk_mean(values):
+    """A chunk's mean as the selection kernel forms it from fp32 scores: the
+    members summed left to right in fp32, divided by the count in fp32.  The
+    exact replay of the GPU's selection on its own scores ranks chunks by this
+    value (the oracle's R18 mean is fp64); the fp64 check of the same kept set
+    then allows the difference near the threshold."""
+    s = np.float32(0.0)
+    for v in values:
+        s = np.float32(s + np.float32(v))
+    return float(np.float32(s / np.float32(len(values))))
+
+
 def oracle_kept(sc, pos, K, P, cap, chunk=1):
-    """The oracle's kept slots: token-level, or chunk-level for chunk > 1."""
+    """The oracle's selection replayed on the GPU's own fp32 scores:
+    token-level, or chunk-level (with the kernel's fp32 chunk mean) for
+    chunk > 1."""
     if chunk > 1:
-        return O.select_kept_chunked(np.asarray(sc, np.float64), pos, K, P, cap, chunk)
+        return O.select_kept_chunked(np.asarray(sc, np.float64), pos, K, P, cap, chunk, mean=kernel_chunk_mean)
     return O.select_kept(np.asarray(sc, np.float64), K, P, cap)
 
 
@@ -384,7 +463,7 @@ def oracle_bandz_at(model, tabs, seq, t, w=64):
     seg = gen.segment_index(model, seq, t + 1)
     z = {}
     for l in model.band_layers:
-        rows = gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg))
+        rows = gen.bf16_bits_to_f64(host.hidden_rows(model, tabs, seq, l, pos, seg))
         g = [O.hidden_change(rows[i - 1], rows[i]) for i in range(1, len(pos))]   # positions lo+1 .. t
         window = g[-min(w, t):]
         z[l] = [O.window_zscore(window)]
@@ -400,7 +479,7 @@ def oracle_hsvar_at(model, tabs, seq, t, w=64):
     seg = gen.segment_index(model, seq, t + 1)
     m = {}
     for l in model.band_layers:
-        rows = gen.bf16_bits_to_f64(gen.hidden_rows(model, tabs, seq, l, pos, seg))
+        rows = gen.bf16_bits_to_f64(host.hidden_rows(model, tabs, seq, l, pos, seg))
         # g[0] stands for position lo (never inside the window), g[j] for lo + j
         g = np.array([np.nan] + [O.hidden_change(rows[i - 1], rows[i]) for i in range(1, len(pos))])
         m[l] = O.rolling_band_mean(g, w)[-1]
@@ -411,7 +490,7 @@ def oracle_kv_at(model, tabs, seq, t, kind, w=64):
     """fp64 KV-key / KV-val score of position t."""
     pos = np.arange(max(0, t - w + 1), t + 1)
     sp = gen.spike_flags(model, seq, t + 1)
-    X = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0 if kind == E.EPIKV_SCORE_KVKEY else 1, pos, sp))
+    X = gen.bf16_bits_to_f64(host.kv_rows(model, tabs, seq, 0 if kind == E.EPIKV_SCORE_KVKEY else 1, pos, sp))
     return float(O.rolling_mean(np.array([O.head_variance(X[i]) for i in range(len(pos))]), w)[-1])
 
 
@@ -431,8 +510,8 @@ def oracle_lag_at(model, tabs, seq, t, lag=16, w=64, key_only=False):
     first = max(0, (t0 // lag - 1) * lag)
     pos = np.arange(first, t + 1)
     sp = gen.spike_flags(model, seq, t + 1)
-    K = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 0, pos, sp))
-    V = gen.bf16_bits_to_f64(gen.kv_rows(model, tabs, seq, 1, pos, sp))
+    K = gen.bf16_bits_to_f64(host.kv_rows(model, tabs, seq, 0, pos, sp))
+    V = gen.bf16_bits_to_f64(host.kv_rows(model, tabs, seq, 1, pos, sp))
     u = []
     for tt in range(t0, t + 1):
         c = tt // lag
@@ -452,8 +531,8 @@ def check_compaction_sampled(sess, b, pos_after, n_rows, rng):
     slots = np.sort(rng.choice(len(pos_after), size=min(n_rows, len(pos_after)), replace=False))
     sp = gen.spike_flags(sess.m, b, int(pos_after.max()) + 1)
     k, v = sess.cache_rows_u16(b, slots)
-    np.testing.assert_array_equal(k, gen.kv_rows(sess.m, sess.dt.tabs, b, 0, pos_after[slots], sp))
-    np.testing.assert_array_equal(v, gen.kv_rows(sess.m, sess.dt.tabs, b, 1, pos_after[slots], sp))
+    np.testing.assert_array_equal(k, host.kv_rows(sess.m, sess.dt.tabs, b, 0, pos_after[slots], sp))
+    np.testing.assert_array_equal(v, host.kv_rows(sess.m, sess.dt.tabs, b, 1, pos_after[slots], sp))
 
 
 def check_compaction(sess, b, pos_after):
@@ -461,5 +540,5 @@ def check_compaction(sess, b, pos_after):
     sp = gen.spike_flags(sess.m, b, int(pos_after.max()) + 1)
     tabs = sess.dt.tabs
     k, v = sess.cache_rows_u16(b, np.arange(len(pos_after)))
-    np.testing.assert_array_equal(k, gen.kv_rows(sess.m, tabs, b, 0, pos_after, sp))
-    np.testing.assert_array_equal(v, gen.kv_rows(sess.m, tabs, b, 1, pos_after, sp))
+    np.testing.assert_array_equal(k, host.kv_rows(sess.m, tabs, b, 0, pos_after, sp))
+    np.testing.assert_array_equal(v, host.kv_rows(sess.m, tabs, b, 1, pos_after, sp))

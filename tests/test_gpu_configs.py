@@ -9,7 +9,10 @@ fp64 oracle:
   slots of sampled sequences equal the generator's rows byte for byte;
 * sampled kept tokens' scores equal the oracle's fp64 score of the same
   position (computed one by one from the rows of its window) within
-  1e-4 * max(1, |s|).
+  1e-4 * max(1, |s|);
+* at one event of one sequence per workload, the kept list against the fp64
+  oracle's scores of every slot of the pre-event cache (threshold ties
+  allowed, as check_selection states).
 Configuration 1 is small enough for the full oracle: every score, the fp64
 kept set and every compacted row are checked.
 """
@@ -64,7 +67,23 @@ def _score_samples(sess, seqs, per_seq, rng, kinds):
                 assert_scores_close([sc[i]], [ref], f"seq {b} kind {kind} position {t}")
 
 
-def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq, select_chunk=1):
+def _fp64_event_check(sess, b, kl, pos, sc, length, wl, select_chunk=1):
+    """The kept list of one sequence at one eviction event against the fp64
+    oracle: its scores of every pre-event slot from the whole trace up to the
+    event (positions < length), then the exact replay on the GPU's scores
+    and the threshold-tie check on the fp64 ones (check_selection)."""
+    kind = sess.policies[b]
+    ref = OracleTrace(sess.m, sess.dt.tabs, b, length, kind, z_window=wl.z_window, lag=wl.lag,
+                      lag_window=wl.lag_window)
+    cond = ref.cond.get(kind)
+    check_selection(kl, pos, sc, ref.scores[kind][pos], wl.budgets[b], sess.prefill[b], sess.recency_cap,
+                    select_chunk, None if cond is None else cond[pos])
+
+
+def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq, select_chunk=1, fp64_event=None):
+    """fp64_event = (step, sequence): the sampled event whose kept list is
+    also checked against the fp64 oracle's scores of the whole pre-event
+    cache."""
     m = wl.model
     rng = np.random.default_rng(wl.model.seed)
     K = wl.budgets[0]
@@ -74,6 +93,7 @@ def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq, select_ch
     triggers = [budgets[b] + wl.trigger_slack[b] for b in range(wl.n_seq)]
     n_steps = wl.max_len // wl.chunk
     events = 0
+    fp64_done = False
     for st in range(n_steps):
         entries = [(b, wl.chunk) for b in range(wl.n_seq)]
         if st in sampled_steps:
@@ -84,10 +104,15 @@ def _run_chunked(wl, sampled_steps, sample_bytes, score_seqs, per_seq, select_ch
             sess.compact(seqs)
             assert len(kept) == wl.n_seq, f"step {st}: expected every sequence to evict"
             _event_checks(sess, pre, kept, budgets, rng, sample_bytes)
+            if fp64_event is not None and fp64_event[0] == st:
+                b = fp64_event[1]
+                _fp64_event_check(sess, b, kept[b], *pre[b], (st + 1) * wl.chunk, wl, select_chunk)
+                fp64_done = True
             events += 1
         else:
             sess.step(entries, budgets, triggers)
     assert events == len(sampled_steps)
+    assert fp64_event is None or fp64_done
     assert all(n == K for n in sess.n_cache)
     _score_samples(sess, score_seqs, per_seq, rng, wl.kinds)
     assert sess.error() == (E.EPIKV_OK, 0)
@@ -121,7 +146,7 @@ def test_config2_batch8_8k_bandz(gpu_lib):
     wl = W.config(2)
     first = wl.budgets[0] // wl.chunk            # the first step that evicts
     _run_chunked(wl, {first, 100, wl.max_len // wl.chunk - 1}, sample_bytes={0, 5}, score_seqs=range(8),
-                 per_seq=6)
+                 per_seq=6, fp64_event=(100, 3))
 
 
 def test_config2_shape_with_chunk_level_selection(gpu_lib):
@@ -130,7 +155,7 @@ def test_config2_shape_with_chunk_level_selection(gpu_lib):
     wl = W.config(2)
     first = wl.budgets[0] // wl.chunk
     _run_chunked(wl, {first, 77, wl.max_len // wl.chunk - 1}, sample_bytes={3}, score_seqs=(2,), per_seq=3,
-                 select_chunk=16)
+                 select_chunk=16, fp64_event=(77, 6))
 
 
 def test_config2_shape_with_all_six_score_kinds(gpu_lib):
@@ -141,14 +166,15 @@ def test_config2_shape_with_all_six_score_kinds(gpu_lib):
     pol = tuple(ALL_KINDS[b % 6] for b in range(wl.n_seq))
     wl = dataclasses.replace(wl, kinds=63, policies=pol)
     first = wl.budgets[0] // wl.chunk
-    _run_chunked(wl, {first, wl.max_len // wl.chunk - 1}, sample_bytes={1, 4}, score_seqs=range(6), per_seq=3)
+    _run_chunked(wl, {first, wl.max_len // wl.chunk - 1}, sample_bytes={1, 4}, score_seqs=range(6), per_seq=3,
+                 fp64_event=(first, 5))
 
 
 def test_config3_batch32_32k_lagkv_paged(gpu_lib):
     wl = W.config(3)
     first = wl.budgets[0] // wl.chunk
     _run_chunked(wl, {first, 150, wl.max_len // wl.chunk - 1}, sample_bytes={0, 17}, score_seqs=(0, 9, 22, 31),
-                 per_seq=4)
+                 per_seq=4, fp64_event=(150, 22))
 
 
 def test_config4_batch4_64k_per_token_updates(gpu_lib):
@@ -201,6 +227,10 @@ def test_config4_batch4_64k_per_token_updates(gpu_lib):
     kept_h = kept.cpu().numpy()
 
     s = _CacheProbe(m, dt, cache, None)
+    # sequence 2's eviction against the fp64 oracle's scores of all 65,536 positions
+    ref = OracleTrace(m, dt.tabs, 2, T, E.EPIKV_SCORE_BANDZ)
+    check_selection(list(kept_h[2]), pre[2][0], pre[2][1], ref.scores[E.EPIKV_SCORE_BANDZ], K, 0, 128, 1,
+                    ref.cond[E.EPIKV_SCORE_BANDZ])
     for b in range(Bn):
         pos, sc = pre[b]
         exp = O.select_kept(sc.astype(np.float64), K, 0, 128)
@@ -252,6 +282,8 @@ def test_config5_ragged_continuous_batch_both_scores(gpu_lib):
     want_events = {b: {0, n_events[b] // 2, n_events[b] - 1} for b in even + odd}
     assert all(n_events[b] >= 3 for b in want_events)
     events_seen = {b: 0 for b in want_events}
+    fp64_seqs = {even[1], odd[1]}     # one band-z-policy and one Lag-KV-policy sequence
+    fp64_checked = set()
     s = _CacheProbe(m, dt, cache, bt)
     total_events = 0
     out = torch.empty(Bn, dtype=torch.int32, device="cuda")
@@ -291,6 +323,14 @@ def test_config5_ragged_continuous_batch_both_scores(gpu_lib):
                 kl = kept_h[i, :K]
                 exp = O.select_kept(pre[b][1].astype(np.float64), K, 0, 128)
                 assert list(kl) == exp, f"seq {b} event: selection differs from the oracle on the GPU's scores"
+                if b in fp64_seqs and events_seen[b] - 1 == n_events[b] // 2:
+                    # the middle event against the fp64 oracle's scores of the whole pre-event cache
+                    ref = OracleTrace(m, dt.tabs, b, t + 1, wl.policies[b])
+                    cond = ref.cond.get(wl.policies[b])
+                    pp = pre[b][0]
+                    check_selection(list(kl), pp, pre[b][1], ref.scores[wl.policies[b]][pp], K, 0, 128, 1,
+                                    None if cond is None else cond[pp])
+                    fp64_checked.add(b)
                 p_after, _, nn = E.epikv_read_slots(ctx, b, wl.policies[b], T_cap)
                 assert nn == K
                 np.testing.assert_array_equal(np.array(p_after), pre[b][0][kl])
@@ -304,6 +344,7 @@ def test_config5_ragged_continuous_batch_both_scores(gpu_lib):
     torch.cuda.synchronize()
     assert total_events > 1000
     assert all(events_seen[b] == n_events[b] for b in want_events)
+    assert fp64_checked == fp64_seqs
     for b in range(Bn):
         p, _, nn = E.epikv_read_slots(ctx, b, 1, 1)
         assert nn == n_cache[b], (b, nn, n_cache[b])

@@ -407,6 +407,21 @@ def _brute_chunked(s, pos, K, P, cap, C):
     return sorted(set(range(P)) | set(range(n - R, n)) | set(valid[0]))
 
 
+def test_chunk_mean_is_the_float64_mean_not_a_float32_one():
+    """R18's chunk score is the members' mean itself: two chunks whose means
+    differ by 2^-32 (indistinguishable once rounded to float32, where the
+    earlier chunk would win the tie) rank by the exact difference, and the
+    mean of members whose float32 running sum loses the small one keeps it."""
+    # slots 0, 1 -> chunk 0 (mean 2); slots 2, 3 -> chunk 1 (mean 2 + 2^-32); slots 4.. recency
+    s = [1.0, 3.0, 2.0 + 2.0 ** -30, 2.0 - 2.0 ** -31, 0.0, 0.0]
+    pos = [0, 1, 2, 3, 4, 5]
+    # K = 4: R = 1 (one recency slot), M = 3 -> chunk 1 whole, then chunk 0's lowest slot
+    assert O.select_kept_chunked(s, pos, 4, 0, 1, 2) == [0, 2, 3, 5]
+    assert np.float32(s[2]) == np.float32(s[3]) == np.float32(2.0)   # a float32 mean would tie at 2
+    assert O.chunk_mean([1e8, 1.0, -1e8]) == pytest.approx(1.0 / 3.0, rel=1e-15)   # float32: 0 / 3
+    assert math.isnan(O.chunk_mean([1.0, float("nan")]))
+
+
 def test_chunked_select_equals_brute_force_on_tiny_inputs():
     rng = np.random.default_rng(22)
     for trial in range(300):

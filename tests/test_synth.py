@@ -72,3 +72,26 @@ def test_pyramid_budgets_recipe():
         assert abs(sum(b) / L - k_mean) <= 8                          # the mean stays K (rounding to 16)
         assert b[0] == round(1.5 * k_mean / 16) * 16 and b[-1] == round(0.5 * k_mean / 16) * 16
     assert W.pyramid_budgets(100, 1) == (96,)
+
+
+def test_host_twin_matches_numpy_generator_byte_for_byte():
+    """The C twin of the generator (used by the oracle's full-size checks)
+    gives the numpy generator's bytes: small and full model shapes, Band A
+    layers with segment jumps, spike positions, unordered positions, another
+    seed and sequence.  Built by the package build; skipped where it is not."""
+    from synth import host
+    if host.load() is None:
+        pytest.skip("libepikv_synth_host.so not built")
+    for m, seq in ((workloads.small_model(11), 0), (gen.TraceModel(0xE91C0003), 5), (gen.TraceModel(99), 2)):
+        tabs = gen.make_tables(m)
+        T = 3000
+        sp = gen.spike_flags(m, seq, T)
+        seg = gen.segment_index(m, seq, T)
+        spike_pos = np.nonzero(sp)[0][:3]
+        pos = np.concatenate([[0, 1, 2, T - 1, 777, 5], spike_pos, spike_pos + 1, np.arange(100, 170)])
+        for kind in (0, 1):
+            np.testing.assert_array_equal(host.kv_rows(m, tabs, seq, kind, pos, sp),
+                                          gen.kv_rows(m, tabs, seq, kind, pos, sp))
+        for layer in sorted({0, m.band_a[0], m.band_b[-1], m.num_layers - 1}):
+            np.testing.assert_array_equal(host.hidden_rows(m, tabs, seq, layer, pos, seg),
+                                          gen.hidden_rows(m, tabs, seq, layer, pos, seg))

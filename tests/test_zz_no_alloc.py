@@ -1,4 +1,5 @@
-"""The allocation-free Lag-KV entry point against the context path.
+"""The allocation-free Lag-KV entry point against the context path and the
+fp64 oracle.
 
 epikv_lagkv_score_noalloc serves callers that cannot allocate device memory
 (no workspace, no context): its scratch is a fixed array inside the library.
@@ -16,7 +17,7 @@ from paper_2606_26472_gb300.cache import KVCache
 from synth import gen
 from synth.device import DeviceTrace
 
-from .harness import assert_scores_close
+from .harness import OracleTrace, assert_scores_close
 
 pytestmark = pytest.mark.gpu
 
@@ -69,9 +70,49 @@ def test_noalloc_scores_match_the_context_path_on_two_calls(gpu_lib):
         got = out[b, :n].cpu().numpy()
         assert_scores_close(got, ref[b], f"no-alloc seq {b}")
         assert np.all(np.isnan(out[b, n:].cpu().numpy()))   # nothing written past n
+    # and both against the fp64 oracle, position by position
+    orc = OracleTrace(model, dt.tabs, 1, lens[1], E.EPIKV_SCORE_LAGKV)
+    assert_scores_close(out[1, :lens[1]].cpu().numpy(), orc.scores[E.EPIKV_SCORE_LAGKV], "no-alloc vs oracle")
 
     # a request larger than the fixed scratch is refused before any launch
     too_many = SCRATCH_FLOATS // (2 * L) + 1
     st = lib.epikv_lagkv_score_noalloc(C.byref(view), 0, too_many, L, H, d, 16, C.c_float(1e-6), 64,
                                        out[0].data_ptr(), stream)
     assert st == E.EPIKV_EINVAL
+
+
+# head shapes at the edges of what the entry point accepts, both layouts, a
+# one-token window, a window that does not divide the tile, the largest
+# window, and lags that do not divide n
+SHAPES = [
+    ("d8_h32_paged_w1_lag5", 32, 8, E.EPIKV_LAYOUT_PAGED, 1, 5, 301),
+    ("d64_h4_contig_w200_lag16", 4, 64, E.EPIKV_LAYOUT_CONTIGUOUS, 200, 16, 517),
+    ("d256_h8_paged_w1024_lag7", 8, 256, E.EPIKV_LAYOUT_PAGED, 1024, 7, 1100),
+    ("d128_h8_contig_w64_lag16", 8, 128, E.EPIKV_LAYOUT_CONTIGUOUS, 64, 16, 777),
+]
+
+
+@pytest.mark.parametrize("name,H,d,layout,window,lag,n", SHAPES, ids=[c[0] for c in SHAPES])
+def test_noalloc_matches_the_oracle(gpu_lib, name, H, d, layout, window, lag, n):
+    lib = gpu_lib
+    model = gen.TraceModel(0xE91C0200 + H * d + window, num_layers=3, hidden=256, num_kv_heads=H, head_dim=d,
+                           band_a=(1,), band_b=(2,))
+    L = model.num_layers
+    T = (n + 15) // 16 * 16 + 16
+    seqs = 2
+    bt = gen.block_permutation(31, seqs * (T // 16)).reshape(seqs, T // 16) if layout else None
+    cache = KVCache(layout, L, H, d, max_seqs=seqs, max_tokens=T, block_table=bt)
+    dt = DeviceTrace(model)
+    dt.kv(1, 0, n, 0, cache.k, cache.v, **cache.synth_kwargs())
+    view = cache.view()
+    out = torch.full((2, T), float("nan"), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    for rep in range(2):       # two calls in a row: the second finds the first's scratch contents
+        st = lib.epikv_lagkv_score_noalloc(C.byref(view), 1, n, L, H, d, lag, C.c_float(1e-6), window,
+                                           out[rep].data_ptr(), stream)
+        assert st == E.EPIKV_OK
+    torch.cuda.synchronize()
+    ref = OracleTrace(model, dt.tabs, 1, n, E.EPIKV_SCORE_LAGKV, lag=lag, lag_window=window)
+    for rep in range(2):
+        assert_scores_close(out[rep, :n].cpu().numpy(), ref.scores[E.EPIKV_SCORE_LAGKV], f"{name} call {rep}")
+        assert np.all(np.isnan(out[rep, n:].cpu().numpy()))
