@@ -299,11 +299,16 @@ epikv_status epikv_get_error(epikv_ctx* ctx, int32_t* code);
  * Working memory is a fixed 2 MiB array inside the library (every GPU that
  * loads the library holds it until the process exits), so n * 2 * L must not
  * exceed 524,288 (n <= 8,192 at L = 32): larger requests return EPIKV_EINVAL
- * and launch nothing.  The first call on each device looks the array's
- * address up (with that device current); make that first call before any
- * stream capture.  All calls share the array: calls that overlap on the GPU
+ * and launch nothing.  The first call in each CUDA context looks the array's
+ * address up (with that context current) and remembers it under the
+ * context's unique id, so a context created again after cudaDeviceReset gets
+ * a fresh lookup; make the first call in a context before any stream
+ * capture.  All calls share the array: calls that overlap on the GPU
  * (unordered streams) race and must be avoided; calls ordered on one stream
- * are independent. */
+ * are independent.  Slots the view does not map (a negative or out-of-range
+ * block-table entry) are read as zero rows and are not reported.  A CUDA
+ * error already pending on the calling thread is returned as EPIKV_ECUDA
+ * before anything is launched, and left in place for its owner. */
 epikv_status epikv_lagkv_score_noalloc(const epikv_kv_view* kv, int32_t seq, int32_t n,
                                        int32_t num_layers, int32_t num_kv_heads, int32_t head_dim,
                                        int32_t lag, float lag_eps, int32_t window, float* d_scores,

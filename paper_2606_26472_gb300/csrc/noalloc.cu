@@ -11,19 +11,28 @@
 // The scratch is `g_noalloc_scratch`, a file-scope static device array of
 // kNoallocScratchFloats floats (2 MiB).  Every GPU that loads the library
 // holds it until the process exits.  In host code that name is only a host
-// stand-in, not a device address: the first call on each device (with that
-// device current) looks the real address up with cudaGetSymbolAddress and
-// remembers it; that set-up is why the first call on a device should come
-// before any stream capture.  The array is shared by every call and keeps the
-// previous call's contents; every entry a call reads is written by the same
-// call first, so nothing needs clearing, but two calls that overlap on the GPU
-// (different streams, no ordering between them) race on it.
+// stand-in, not a device address: the first call in each CUDA context (with
+// that context's device current) looks the real address up with
+// cudaGetSymbolAddress and remembers it under the context's unique id, so a
+// context that is torn down and created again (cudaDeviceReset) gets a fresh
+// lookup instead of a stale address; that set-up is why the first call in a
+// context should come before any stream capture.  The array is shared by
+// every call and keeps the previous call's contents; every entry a call reads
+// is written by the same call first, so nothing needs clearing, but two calls
+// that overlap on the GPU (different streams, no ordering between them) race
+// on it.
+//
+// Slots the view does not map (a negative or out-of-range block-table entry)
+// are read as zero rows: this entry point has no error word, so such input
+// is not reported.
 //
 // The kernels are variants of the Lag-KV partial and finalize kernels of the
 // context path, for a sequence whose slots 0..n-1 hold positions 0..n-1.  They
 // take each head's variance in two passes (mean, then squared deviations),
 // where the context path uses shifted moments in one pass, so the scores agree
 // with epikv_score_update's to fp32 rounding, not bit for bit.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -31,7 +40,7 @@
 namespace {
 
 constexpr size_t kNoallocScratchFloats = size_t(1) << 19;  // 2 MiB: n * 2 * num_layers floats
-constexpr int kMaxDevices = 64;
+constexpr int kMaxContexts = 64;  // contexts whose scratch address is remembered
 constexpr int kBatch = 16;
 constexpr int kTile = 32;
 constexpr int kThreads = 256;
@@ -162,23 +171,60 @@ __global__ void __launch_bounds__(kThreads) noalloc_finalize_kernel(const float*
   }
 }
 
-std::mutex g_mu;
-float* g_scratch_ptr[kMaxDevices] = {};
+// The current context's unique id (driver entry points fetched through the
+// runtime, so the library needs no link-time dependency on the driver).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
 
-// Device address of the scratch array on the current device (looked up once).
-cudaError_t scratch_address(float** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+std::mutex g_mu;
+CtxGetCurrentFn g_ctx_current = nullptr;
+CtxGetIdFn g_ctx_id = nullptr;
+struct ScratchEntry {
+  unsigned long long ctx_id;
+  float* ptr;
+};
+ScratchEntry g_scratch[kMaxContexts] = {};
+int g_scratch_next = 0;
+
+cudaError_t current_context_id(unsigned long long* id) {
+  if (!g_ctx_current || !g_ctx_id) {
+    void* f1 = nullptr;
+    void* f2 = nullptr;
+    cudaDriverEntryPointQueryResult q1, q2;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f1, 12000, cudaEnableDefault, &q1);
+    if (e == cudaSuccess) e = cudaGetDriverEntryPointByVersion("cuCtxGetId", &f2, 12000, cudaEnableDefault, &q2);
     if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev] = static_cast<float*>(p);
+    if (q1 != cudaDriverEntryPointSuccess || q2 != cudaDriverEntryPointSuccess || !f1 || !f2)
+      return cudaErrorNotSupported;
+    g_ctx_current = reinterpret_cast<CtxGetCurrentFn>(f1);
+    g_ctx_id = reinterpret_cast<CtxGetIdFn>(f2);
   }
-  *out = g_scratch_ptr[dev];
+  CUcontext ctx = nullptr;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || !ctx) return cudaErrorDeviceUninitialized;
+  return g_ctx_id(ctx, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorContextIsDestroyed;
+}
+
+// Device address of the scratch array in the current context: looked up once
+// per context, then taken from the table.
+cudaError_t scratch_address(float** out) {
+  std::lock_guard<std::mutex> lock(g_mu);
+  unsigned long long id = 0;
+  if (current_context_id(&id) == cudaSuccess)
+    for (const ScratchEntry& s : g_scratch)
+      if (s.ptr && s.ctx_id == id) {
+        *out = s.ptr;
+        return cudaSuccess;
+      }
+  // first call in this context (this also makes the device's primary context
+  // current if no context was yet)
+  void* p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess) return e;
+  e = current_context_id(&id);
+  if (e != cudaSuccess) return e;
+  g_scratch[g_scratch_next] = ScratchEntry{id, static_cast<float*>(p)};
+  g_scratch_next = (g_scratch_next + 1) % kMaxContexts;
+  *out = static_cast<float*>(p);
   return cudaSuccess;
 }
 
@@ -223,6 +269,9 @@ extern "C" epikv_status epikv_lagkv_score_noalloc(const epikv_kv_view* kv, int32
   if ((size_t)n * 2 * (size_t)L > kNoallocScratchFloats) return EPIKV_EINVAL;  // beyond the fixed scratch
   KvDev kd;
   if (!view_ok(kv, H, d, &kd)) return EPIKV_EINVAL;
+  // an error left by earlier, unrelated work stays with its owner: report it
+  // without launching and without clearing it
+  if (cudaPeekAtLastError() != cudaSuccess) return EPIKV_ECUDA;
   float* part = nullptr;
   if (scratch_address(&part) != cudaSuccess) return EPIKV_ECUDA;
 
@@ -248,5 +297,6 @@ extern "C" epikv_status epikv_lagkv_score_noalloc(const epikv_kv_view* kv, int32
     noalloc_finalize_kernel<8><<<g2, kThreads, 0, stream>>>(part, n, L, H, lag, window, d_scores);
   else
     noalloc_finalize_kernel<32><<<g2, kThreads, 0, stream>>>(part, n, L, H, lag, window, d_scores);
+  // no error was pending before the launches, so any error now is theirs
   return cudaGetLastError() == cudaSuccess ? EPIKV_OK : EPIKV_ECUDA;
 }
