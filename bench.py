@@ -1,13 +1,14 @@
 #!/usr/bin/env python
 """Throughput of the EpiKV eviction hot path on GB300.
 
-Workload (the 32k-context decode configuration): 32 sequences, 32 layers x 8
-KV heads x 128 dims bf16 K/V in a paged pool of 16-token blocks with shuffled
-block tables, budget K = 8192, Lag-KV scores (lag 16, rolling window 64).
-One step = the steady-state decode chunk of every sequence: 128 new tokens
-per sequence are scored, each cache (8,320 tokens) is cut back to K and every
-layer's K and V are compacted in place -- one epikv_step through the C ABI
-(Lag-KV partial kernel, finalize kernel, select kernel, TMA compaction kernel).
+Headline workload (the 32k-context decode configuration): 32 sequences per
+GPU, 32 layers x 8 KV heads x 128 dims bf16 K/V in a paged pool of 16-token
+blocks with shuffled block tables, budget K = 8192, Lag-KV scores (lag 16,
+rolling window 64).  One step = the steady-state decode chunk of every
+sequence: 128 new tokens per sequence are scored, each cache (8,320 tokens)
+is cut back to K and every layer's K and V are compacted in place -- one
+epikv_step through the C ABI (Lag-KV partial kernel, finalize kernel, select
+kernel, TMA compaction kernel).
 
 Inputs are resident in HBM before timing: the 8,192-token caches and the new
 tokens of every timed step (pre-generated into fresh pool blocks that each
@@ -15,11 +16,16 @@ step's block table points to, as a paged serving loop appends tokens).  The
 cache and pool (tens of GB) are far larger than L2, so no flush is needed.
 
 `value` = tokens scored per second over the timed steps (all ranks);
-`e2e` = the same through the same call with the new tokens' K/V copied from
-pinned host memory every step and the new cache lengths read back;
+`e2e` = the same steps again through the same call, from the same state (the
+workspace and resident caches are restored), with each step's new K/V copied
+from pinned host memory and the new cache lengths read back;
 `roofline` = the compaction kernel's algorithmic bytes (2 x moved rows x
 128 KiB) per launch over its CUDA-event duration, against the measured HBM
-copy bandwidth.  `--impl reference` times the fp64 CPU oracle instead.
+copy bandwidth; `configs` = the five workloads measured one after another
+(single GPU), each with its kernels' CUDA-event times and HBM fractions.
+Under torchrun every rank owns its own sequences (global ids rank * 32 ..
+rank * 32 + 31): the batch is sharded by sequence with no data exchange.
+`--impl reference` times the fp64 CPU oracle instead.
 """
 from __future__ import annotations
 
@@ -42,48 +48,66 @@ UNIT = "tokens/s"
 WORKLOAD = "batch32_32k_lagkv_paged16_K8192_chunk128"
 
 
-def parse():
+def parse(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    # end-to-end steps, each with its own 512 MiB of new K/V in pinned host memory
-    p.add_argument("--e2e-steps", type=int, default=50)
+    # skip the per-configuration table of the default run
+    p.add_argument("--no-configs", action="store_true")
     # CTAs of the end-to-end measurement's host-to-device upload kernel
     p.add_argument("--upload-ctas", type=int, default=32)
     # a scaled-down variant of the same workload, for profiler captures
     p.add_argument("--sequences", type=int, default=32)
     p.add_argument("--budget", type=int, default=8192)
     p.add_argument("--chunk", type=int, default=128)
-    # the band-z kernels' workload: the 2,048-token single-sequence case, one
-    # fresh sequence per step (reported for the per-kernel rooflines)
-    p.add_argument("--workload", default="lagkv32k", choices=["lagkv32k", "bandz2k", "pertoken", "layers32k", "bandz8k", "ragged64"])
+    # one workload alone (the per-configuration table runs them all):
+    # bandz2k = configuration 1, bandz8k = 2, lagkv32k = 3 (default),
+    # pertoken / evict64k = the two phases of 4, ragged64 = 5; layers32k =
+    # per-layer budgets on configuration 3's shape
+    p.add_argument("--workload", default="lagkv32k",
+                   choices=["lagkv32k", "bandz2k", "pertoken", "evict64k", "layers32k", "bandz8k", "ragged64"])
     # K/V score kinds computed at the 32k workload (selection uses Lag-KV):
     # 2 = Lag-KV only; 58 = Lag-KV + KV-key + KV-val + lag-kv-key
     p.add_argument("--kinds", type=int, default=2)
     # chunk-level selection at the 32k workload: position chunks of this many
     # tokens (1 = the paper's token-level selection)
     p.add_argument("--select-chunk", type=int, default=1)
-    return p.parse_args()
+    # oracle processes of the CPU baseline (0: one per available core)
+    p.add_argument("--cpu-workers", type=int, default=0)
+    return p.parse_args(argv)
 
 
 def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
 
 
+def shard_sequences(per_rank, rank, world):
+    """Global sequence ids owned by `rank` when a batch of per_rank * world
+    sequences is split by sequence over `world` ranks: a contiguous block of
+    per_rank ids.  Every sequence (its K/V, its workspace slots, its seeds)
+    lives on exactly one rank, so ranks exchange no data."""
+    assert 0 <= rank < world and per_rank >= 1
+    return list(range(rank * per_rank, (rank + 1) * per_rank))
+
+
 def aggregate_ranks(local_ms, units_per_rank, world, device=None):
-    """Whole-job timing of weak-scaling replicas: the slowest rank's duration
+    """Whole-job timing of sequence-sharded ranks: the slowest rank's duration
     and the units all ranks processed per second over it."""
+    units = float(units_per_rank)
     if world > 1:
         import torch
         import torch.distributed as dist
         t = torch.tensor([local_ms], dtype=torch.float64, device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         local_ms = float(t.item())
-    return local_ms, world * units_per_rank / (local_ms / 1e3)
+        u = torch.tensor([units], dtype=torch.float64, device=device)
+        dist.all_reduce(u, op=dist.ReduceOp.SUM)
+        units = float(u.item())
+    return local_ms, units / (local_ms / 1e3)
 
 
 def measured_hbm_peak():
@@ -141,6 +165,7 @@ class Clocks:
         except Exception:
             self.proc = None
         time.sleep(0.3)
+        return self
 
     def stop(self):
         if self.proc is None:
@@ -165,106 +190,220 @@ class Clocks:
 
 
 # --------------------------------------------------------------------------- CPU oracle
-def oracle_step_sample(n_seqs, pos0):
-    """Time the fp64 oracle on `n_seqs` sequence-steps of the workload: Lag-KV
-    scores of 128 new tokens, full-sort selection over the 8,320-slot cache and
-    the gather of the kept K/V rows.  Returns (tokens, seconds)."""
+def oracle_sequence_step(seq, pos0):
+    """One sequence's decode step of the 32k workload, timed on the fp64
+    oracle: Lag-KV scores of 128 new tokens, full-sort selection over the
+    8,320-slot cache and the gather of the kept K/V rows of every layer.  The
+    rows are regenerated first, untimed.  Returns (tokens, seconds)."""
     from oracle import epikv_oracle as O
-    from synth import gen, workloads as W
+    from synth import gen, host, workloads as W
 
     wl = W.config(3)
     m = wl.model
     tabs = gen.make_tables(m)
     K, C, lag, w = wl.budgets[0], wl.chunk, wl.lag, wl.lag_window
-    n_slots = K + C
-    shape = (n_slots, m.num_layers, m.num_kv_heads, m.head_dim)
+    shape = (K + C, m.num_layers, m.num_kv_heads, m.head_dim)
     cache_k = np.ones(shape, np.uint16)       # gather cost does not depend on the bytes
     cache_v = np.ones(shape, np.uint16)
     first = (pos0 - (w - 1)) // lag * lag - lag  # rows the u window and its ranges reach
     positions = np.arange(first, pos0 + C)
-    elapsed = 0.0
-    tokens = 0
-    for b in range(n_seqs):
-        sp = gen.spike_flags(m, b, pos0 + C)
-        Kr = gen.bf16_bits_to_f64(gen.kv_rows(m, tabs, b, 0, positions, sp))
-        Vr = gen.bf16_bits_to_f64(gen.kv_rows(m, tabs, b, 1, positions, sp))
-        old = np.random.default_rng(b).normal(size=K)   # frozen scores of the cached tokens
-        t0 = time.perf_counter()
-        u = {}
-        for t in range(pos0 - (w - 1), pos0 + C):
-            c = t // lag
-            lo = (c - 1) * lag - first
-            u[t] = O.lag_token_variance(Kr[t - first], Vr[t - first], Kr[lo:lo + lag], Vr[lo:lo + lag])
-        s_new = [np.mean([u[t - k] for k in range(w)]) for t in range(pos0, pos0 + C)]
-        scores = np.concatenate([old, s_new])
-        kept = O.select_kept(scores, K, 0, wl.recency_cap)
-        O.compact(cache_k, kept)
-        O.compact(cache_v, kept)
-        elapsed += time.perf_counter() - t0
-        tokens += C
-    return tokens, elapsed
+    sp = gen.spike_flags(m, seq, pos0 + C)
+    Kr = gen.bf16_bits_to_f64(host.kv_rows(m, tabs, seq, 0, positions, sp))
+    Vr = gen.bf16_bits_to_f64(host.kv_rows(m, tabs, seq, 1, positions, sp))
+    old = np.random.default_rng(seq).normal(size=K)   # frozen scores of the cached tokens
+    t0 = time.perf_counter()
+    u = {}
+    for t in range(pos0 - (w - 1), pos0 + C):
+        c = t // lag
+        lo = (c - 1) * lag - first
+        u[t] = O.lag_token_variance(Kr[t - first], Vr[t - first], Kr[lo:lo + lag], Vr[lo:lo + lag])
+    s_new = [np.mean([u[t - k] for k in range(w)]) for t in range(pos0, pos0 + C)]
+    scores = np.concatenate([old, s_new])
+    kept = O.select_kept(scores, K, 0, wl.recency_cap)
+    O.compact(cache_k, kept)
+    O.compact(cache_v, kept)
+    return C, time.perf_counter() - t0
 
 
-def cpu_baseline(target_s=12.0):
-    n = 1
-    tok, sec = oracle_step_sample(1, 8192 + 128)
-    while sec < target_s and n < 32:
-        more = min(32 - n, max(1, int((target_s - sec) / max(sec / n, 1e-3))))
-        t2, s2 = oracle_step_sample(more, 8192 + 128)
-        tok, sec, n = tok + t2, sec + s2, n + more
-    return {"value": tok / sec, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n} of 32 sequences x 1 decode step (128 tokens: fp64 Lag-KV u over 191 positions + "
+def _oracle_task(job):
+    os.environ.setdefault("OMP_NUM_THREADS", "1")
+    seq, pos0 = job
+    tok, sec = oracle_sequence_step(seq, pos0)
+    return os.getpid(), tok, sec
+
+
+def oracle_workers(requested=0):
+    n = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    return max(1, min(n, requested) if requested else n)
+
+
+def oracle_pool(workers):
+    """A pool of oracle processes (spawn: safe after CUDA use in this process)."""
+    import multiprocessing as mp
+    return mp.get_context("spawn").Pool(workers, initializer=_pool_init)
+
+
+def oracle_batch(pool, jobs):
+    """Oracle sequence-steps on the pool's processes.  Returns (tokens,
+    seconds): the tokens of every job over the busiest process's summed
+    compute time (the processes run concurrently)."""
+    res = pool.map(_oracle_task, jobs, chunksize=1)
+    busy = {}
+    for pid, _, sec in res:
+        busy[pid] = busy.get(pid, 0.0) + sec
+    return sum(t for _, t, _ in res), max(busy.values())
+
+
+def _pool_init():
+    # one core per process: numpy's own threads would oversubscribe the host
+    os.environ["OMP_NUM_THREADS"] = "1"
+    os.environ["OPENBLAS_NUM_THREADS"] = "1"
+    sys.path.insert(0, ROOT)
+
+
+def cpu_baseline(requested_workers=0):
+    """The fp64 oracle on the host's cores: the decode step of all 32 sequences
+    of the 32k workload (one process per core, one sequence-step per task)."""
+    workers = oracle_workers(requested_workers)
+    with oracle_pool(workers) as pool:
+        oracle_batch(pool, [(b, 8192) for b in range(workers)])          # warm-up: imports, first allocations
+        tok, sec = oracle_batch(pool, [(b, 8192 + 128) for b in range(32)])
+    return {"value": tok / sec, "unit": UNIT, "cores": workers, "kind": "oracle",
+            "sample": f"32 of 32 sequences x 1 decode step (128 tokens each: fp64 Lag-KV u over 191 positions + "
                       f"rolling mean, full-sort selection over 8320 slots, gather of the 8192 kept K and V rows "
-                      f"of 32 layers), {sec:.1f} s of single-threaded numpy"}
+                      f"of 32 layers), numpy, one process per core on {workers} cores, rows generated untimed; "
+                      f"time = the busiest process's compute, {sec:.1f} s"}
 
 
 def run_reference(args):
     rank, _, world = dist_env()
     if rank != 0:
-        return
-    budget_s = 180.0
-    tok, sec = oracle_step_sample(1, 8192 + 128)   # one warm-up sample
-    steps = max(1, min(args.steps, int(budget_s / max(sec, 1e-3))))
-    tot_tok, tot_s = 0, 0.0
-    for i in range(steps):
-        t, s = oracle_step_sample(1, 8192 + 128 * (i + 2))
-        tot_tok += t
-        tot_s += s
+        return None
+    workers = oracle_workers(args.cpu_workers)
+    budget_s = 150.0
+    tot_tok, tot_s, steps = 0, 0.0, 0
+    with oracle_pool(workers) as pool:
+        oracle_batch(pool, [(b, 8192) for b in range(workers)])          # warm-up
+        t0 = time.perf_counter()
+        for i in range(max(1, args.steps)):
+            t, s = oracle_batch(pool, [(b, 8192 + 128 * (i + 1)) for b in range(32)])
+            tot_tok += t
+            tot_s += s
+            steps += 1
+            if time.perf_counter() - t0 > budget_s:
+                break
     v = tot_tok / tot_s
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
             "steps": steps, "warmup": 1, "ms_per_step": 1e3 * tot_s / steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "oracle_step": "one sequence's decode step"},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{steps} sequence-steps of the workload, single-threaded numpy fp64"},
+            "config": {"workload": WORKLOAD, "oracle_step": "the decode step of all 32 sequences"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": workers, "kind": "oracle",
+                             "sample": f"{steps} decode steps of the 32 sequences, numpy fp64, one process per "
+                                       f"core on {workers} cores"},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+    return line
 
 
-# --------------------------------------------------------------------------- GPU arm
+# --------------------------------------------------------------------------- GPU helpers
+def gpu_device(local_rank=0):
+    import torch
+
+    from paper_2606_26472_gb300 import build as B
+    from paper_2606_26472_gb300 import epikv as E
+    torch.cuda.set_device(local_rank)
+    if not os.path.exists(E.LIB_PATH):
+        B.build()
+    E.load()
+    return torch.device("cuda", local_rank)
+
+
+def stream_bytes(m, *, tokens, seq_calls, rows_moved, kinds, one_token):
+    """Algorithmic HBM bytes of the streaming kernels over a pass that scored
+    `tokens` tokens in `seq_calls` (sequence, call) pairs and moved
+    `rows_moved` token rows (all layers' K and V):
+    * a token's band rows (15 x 4096 bf16) are read once; a chunked call also
+      reads and writes each sequence's saved previous rows (h_prev), a
+      one-token call reads its new rows and h_prev and writes h_prev;
+    * a token's K and V rows of every layer are read once; with a Lag-KV kind
+      each (sequence, call) also reads and writes its range state
+      ([L][K|V][4][H][d] bf16);
+    * the compaction reads and writes every moved row."""
+    nb, D = len(m.band_layers), m.hidden
+    L, H, d = m.num_layers, m.num_kv_heads, m.head_dim
+    band_row = nb * D * 2
+    kv_row = L * 2 * H * d * 2
+    rng_state = L * 2 * 4 * H * d * 2
+    band = bool(kinds & (1 | 4))
+    kv = bool(kinds & (2 | 8 | 16 | 32))
+    state = 2 * rng_state if kinds & (2 | 32) else 0
+    out = {"compact_kernel": 2 * rows_moved * kv_row}
+    if one_token:
+        if kv:
+            out["token_kernel"] = seq_calls * ((3 * band_row if band else 0) + kv_row + state)
+        elif band:
+            out["bandz_token_kernel"] = seq_calls * 3 * band_row
+    else:
+        if band:
+            out["bandz_g_kernel"] = tokens * band_row + seq_calls * 2 * band_row
+        if kv:
+            out["lagkv_partial_kernel"] = tokens * kv_row + seq_calls * state
+    return out
+
+
+def kernel_table(records, n_steps, bytes_per_pass, peak):
+    """Per-kernel CUDA-event times of a pass of n_steps steps (records: [(name,
+    ms)] from epikv_set_kernel_events) -> {kernel: launches and ms per step,
+    and for the HBM-streaming kernels their algorithmic GB/s and fraction of
+    the measured copy bandwidth}."""
+    from paper_2606_26472_gb300 import epikv as E
+    acc = {}
+    for name, ms in records:
+        a = acc.setdefault(E.kernel_short_name(name), [0, 0.0])
+        a[0] += 1
+        a[1] += ms
+    tab = {}
+    for k, (n, ms) in acc.items():
+        e = {"launches_per_step": n / n_steps, "ms_per_step": ms / n_steps}
+        b = bytes_per_pass.get(k)
+        if b and ms > 0:
+            gbs = b / (ms / 1e3) / 1e9
+            e.update(algorithmic_bytes_per_step=b / n_steps, gbs=gbs, hbm_frac=gbs / peak)
+        tab[k] = e
+    return tab
+
+
+def kernel_pass(E, ctx, n_launches, run):
+    """Run `run()` with every kernel of `ctx` bracketed by events; [(name, ms)]."""
+    kc = E.KernelClock(ctx, n_launches)
+    kc.start()
+    try:
+        run()
+    finally:
+        recs = kc.stop()
+    return recs
+
+
+# --------------------------------------------------------------------------- configuration 3 (headline)
 def run_ours(args):
     import torch
     import torch.distributed as dist
 
-    from paper_2606_26472_gb300 import build as B
     from paper_2606_26472_gb300 import epikv as E
     from paper_2606_26472_gb300.cache import KVCache
     from synth import gen, workloads as W
-    from synth.device import DeviceTrace
+    from synth.device import DeviceTrace, upload_2d
 
     rank, local_rank, world = dist_env()
     if world > 1:
         dist.init_process_group("nccl")
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if not os.path.exists(E.LIB_PATH):
-        B.build()
-    E.load()
+    dev = gpu_device(local_rank)
 
     wl = W.config(3)
     m = wl.model
     Bn, K, C = args.sequences, args.budget, args.chunk
     assert K % wl.block_size == 0 and C % wl.block_size == 0
+    gids = shard_sequences(Bn, rank, world)     # this rank's global sequence ids (generator seeds)
     workload = WORKLOAD if (Bn, K, C) == (wl.n_seq, wl.budgets[0], wl.chunk) else \
         f"batch{Bn}_lagkv_paged16_K{K}_chunk{C}"
     if args.kinds != E.EPIKV_SCORE_LAGKV:
@@ -277,9 +416,10 @@ def run_ours(args):
     mb = T_cap // bs
     common = K // bs
     fresh = C // bs
-    n_steps = args.warmup + args.steps
-    e2e_steps = 0 if args.no_e2e else args.e2e_steps
-    n_blocks = Bn * common + n_steps * Bn * fresh + (2 * Bn * fresh if e2e_steps else 0)
+    kc_steps = 3                                  # the per-kernel pass after the timed steps
+    n_steps = args.warmup + args.steps + kc_steps
+    e2e_on = not args.no_e2e
+    n_blocks = Bn * common + n_steps * Bn * fresh + (2 * Bn * fresh if e2e_on else 0)
     perm = gen.block_permutation(m.seed ^ rank, Bn * common).reshape(Bn, common)
 
     def table(fresh_base):
@@ -307,7 +447,7 @@ def run_ours(args):
 
     # the first K tokens of every trace, scored in decode chunks (no eviction yet)
     for b in range(Bn):
-        dt.kv(b, 0, K, 0, cache.k, cache.v, **cache.synth_kwargs(tables[0]))
+        dt.kv(gids[b], 0, K, 0, cache.k, cache.v, **cache.synth_kwargs(tables[0]))
     seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
     cu_new = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * C).contiguous()
     view0 = cache.view(tables[0])
@@ -316,7 +456,7 @@ def run_ours(args):
     # every step's new tokens, appended into fresh blocks before timing
     for st in range(n_steps):
         for b in range(Bn):
-            dt.kv(b, K + st * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tables[st]))
+            dt.kv(gids[b], K + st * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tables[st]))
     views = [cache.view(t) for t in tables]
     budget = torch.full((Bn,), K, dtype=torch.int32, device=dev)
     trigger = torch.full((Bn,), K + C - 1, dtype=torch.int32, device=dev)
@@ -325,12 +465,17 @@ def run_ours(args):
     st_, code = E.epikv_get_error(ctx)
     assert st_ == E.EPIKV_OK, f"device error {code} during set-up"
 
-    def step(st, view):
+    def step(view):
         E.epikv_step(ctx, Bn, seq_ids, cu_new, C, budget, trigger, None, view, n_out)
 
     for st in range(args.warmup):
-        step(st, views[st])
+        step(views[st])
     torch.cuda.synchronize()
+    # the state before the timed steps, restored for the end-to-end pass so that
+    # it repeats the same steps (same kept lists, same rows moved)
+    snap = None
+    if e2e_on:
+        snap = (ws.clone(), cache.k[:, :Bn * common].clone(), cache.v[:, :Bn * common].clone())
     stats0 = E.epikv_get_stats(ctx)
 
     def new_events():
@@ -342,16 +487,14 @@ def run_ours(args):
     phase = [new_events() for _ in range(args.steps)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    gpu_id = Clocks.device_id(dev, local_rank)
-    clocks = Clocks(gpu_id)
-    clocks.start()
+    clocks = Clocks(Clocks.device_id(dev, local_rank)).start()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     t_start.record(stream)
     for i in range(args.steps):
         E.epikv_set_phase_events(ctx, phase[i])
-        step(args.warmup + i, views[args.warmup + i])
+        step(views[args.warmup + i])
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -371,40 +514,54 @@ def run_ours(args):
     assert tokens == Bn * C * args.steps
     row_bytes = L * 2 * H * d * 2                       # one token's K and V, all layers
     compact_bytes = 2 * rows_moved * row_bytes           # read + write
-    score_bytes = tokens * row_bytes + args.steps * Bn * 2 * (L * 2 * 4 * H * d * 2)  # rows + range state r/w
+    score_bytes = sum(stream_bytes(m, tokens=tokens, seq_calls=Bn * args.steps, rows_moved=0, kinds=args.kinds,
+                                   one_token=False).values())
+    peak, peak_src = measured_hbm_peak()
+
+    # per-kernel CUDA-event times: the next kc_steps steps, every kernel bracketed by events
+    s_k0 = E.epikv_get_stats(ctx)
+    recs = kernel_pass(E, ctx, 8 * kc_steps, lambda: [step(views[args.warmup + args.steps + j])
+                                                      for j in range(kc_steps)])
+    s_k1 = E.epikv_get_stats(ctx)
+    kernels = kernel_table(recs, kc_steps,
+                           stream_bytes(m, tokens=Bn * C * kc_steps, seq_calls=Bn * kc_steps,
+                                        rows_moved=s_k1["rows_moved"] - s_k0["rows_moved"], kinds=args.kinds,
+                                        one_token=False), peak)
 
     ms, value = aggregate_ranks(ms, tokens, world, dev)
 
-    # ---- end to end: new tokens' K/V from pinned host memory, new lengths back
+    # ---- end to end: the timed steps again, from the same state, with each
+    # step's new K/V copied from pinned host memory and its new lengths read back
     e2e = None
-    if e2e_steps:
+    if e2e_on:
+        ws.copy_(snap[0])
+        cache.k[:, :Bn * common].copy_(snap[1])
+        cache.v[:, :Bn * common].copy_(snap[2])
+        del snap
         # two sets of fresh blocks: step i+1's K/V are copied in on a side
         # stream while step i runs, as a serving loop would overlap them
         tabs = [table(e2e_base + j * Bn * fresh) for j in range(2)]
         views_e = [cache.view(t) for t in tabs]
-        # every step's own new tokens (fresh positions, as in the timed loop),
-        # one pinned buffer per step
+        n_e = args.steps
         payload = [torch.empty((2, L, Bn * fresh, bs, H, d), dtype=torch.bfloat16, pin_memory=True)
-                   for _ in range(e2e_steps)]
-        pos_base = K + n_steps * C
+                   for _ in range(n_e)]
         lo = e2e_base
-        for j in range(e2e_steps):
+        for j in range(n_e):     # timed step j's new tokens, generated again, kept on the host
             for b in range(Bn):
-                dt.kv(b, pos_base + j * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tabs[0]))
+                dt.kv(gids[b], K + (args.warmup + j) * C, C, K, cache.k, cache.v, **cache.synth_kwargs(tabs[0]))
             payload[j][0].copy_(cache.k[:, lo:lo + Bn * fresh])
             payload[j][1].copy_(cache.v[:, lo:lo + Bn * fresh])
-        lens = torch.empty((e2e_steps, Bn), dtype=torch.int32, pin_memory=True)
+        lens = torch.empty((n_e, Bn), dtype=torch.int32, pin_memory=True)
         copy_stream = torch.cuda.Stream(device=dev)
-        copied = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        stepped = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        copy_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        step_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+        copied = [torch.cuda.Event(enable_timing=True) for _ in range(n_e)]
+        stepped = [torch.cuda.Event(enable_timing=True) for _ in range(n_e)]
+        copy_start = [torch.cuda.Event(enable_timing=True) for _ in range(n_e)]
+        step_start = [torch.cuda.Event(enable_timing=True) for _ in range(n_e)]
 
         # one strided upload per K and V and step (32 layer planes of 8 MiB
         # each), read from the pinned host buffer by SM loads over the host
         # link: the copy engines of this platform stall every ~0.5 s for
         # ~0.1 s, the SM path does not (both move ~210 GB/s otherwise)
-        from synth.device import upload_2d
         plane = Bn * fresh * bs * H * d * 2                 # bytes of one layer's new rows
         pitch = cache.k.stride(0) * 2                       # bytes between layer planes of the pool
         up_ctas = args.upload_ctas
@@ -428,38 +585,44 @@ def run_ours(args):
         e0.record(stream)
         copy_stream.wait_event(e0)
         h2d(0)
-        for i in range(e2e_steps):
-            if i + 1 < e2e_steps:
+        for i in range(n_e):
+            if i + 1 < n_e:
                 h2d(i + 1)
             stream.wait_event(copied[i])
             step_start[i].record(stream)
-            step(None, views_e[i % 2])
+            step(views_e[i % 2])
             stepped[i].record(stream)
             lens[i].copy_(n_out, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
-        e_ms, e_value = aggregate_ranks(e0.elapsed_time(e1), Bn * C * e2e_steps, world, dev)
+        stats_e1 = E.epikv_get_stats(ctx)
+        e_tokens = stats_e1["tokens_scored"] - stats_e0["tokens_scored"]
+        e_ms, e_value = aggregate_ranks(e0.elapsed_time(e1), e_tokens, world, dev)
         assert (lens.numpy() == K).all()
-        copy_ms = sorted(copy_start[i].elapsed_time(copied[i]) for i in range(e2e_steps))
-        step_ms = sorted(step_start[i].elapsed_time(stepped[i]) for i in range(e2e_steps))
+        copy_ms = sorted(copy_start[i].elapsed_time(copied[i]) for i in range(n_e))
+        step_ms = sorted(step_start[i].elapsed_time(stepped[i]) for i in range(n_e))
+        rows_e = stats_e1["rows_moved"] - stats_e0["rows_moved"]
         e2e = {"value": e_value, "unit": UNIT,
                "h2d_bytes_per_step": int(payload[0].numel() * 2), "d2h_bytes_per_step": Bn * 4,
-               "steps": e2e_steps,
+               "steps": n_e,
+               "same_steps_as_timed": "the timed steps repeated from the restored pre-timing state",
                "overlap": "step i+1's host-to-device upload (SM loads of pinned host memory) runs on a side stream "
                           "during step i",
                "median_ms": {"h2d_copy": copy_ms[len(copy_ms) // 2], "step": step_ms[len(step_ms) // 2],
-                             "wall_per_step": e_ms / e2e_steps},
+                             "wall_per_step": e_ms / n_e},
                "max_ms": {"h2d_copy": copy_ms[-1], "step": step_ms[-1]},
                "slow_copies": sum(c > 2 * copy_ms[len(copy_ms) // 2] for c in copy_ms),
-               "rows_moved_per_step": (E.epikv_get_stats(ctx)["rows_moved"] - stats_e0["rows_moved"]) / e2e_steps}
+               "rows_moved_per_step": rows_e / n_e,
+               "rows_moved_match_timed": rows_e == rows_moved}
         st_, code = E.epikv_get_error(ctx)
         assert st_ == E.EPIKV_OK, f"device error {code} in e2e"
+        del payload
 
+    E.epikv_destroy(ctx)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
-        return
-    peak, peak_src = measured_hbm_peak()
+        return None
     ach = compact_bytes / args.steps / (t_compact / args.steps / 1e3) / 1e9
     ratio = ncu_traffic("compact_kernel")
     traffic = None if ratio is None else ratio * compact_bytes / args.steps
@@ -467,55 +630,57 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": workload, "sequences": Bn, "context": 32768, "budget_K": K, "chunk": C,
-                   "layers": L, "kv_heads": H, "head_dim": d, "kv_dtype": "bf16", "layout": "paged16_shuffled",
-                   "score": "lagkv_lag16_w64", "select_chunk": args.select_chunk,
-                   "parallelism": f"replicas{world}",
+        "config": {"workload": workload, "sequences": Bn, "global_batch": Bn * world, "context": 32768,
+                   "budget_K": K, "chunk": C, "layers": L, "kv_heads": H, "head_dim": d, "kv_dtype": "bf16",
+                   "layout": "paged16_shuffled", "score": "lagkv_lag16_w64", "select_chunk": args.select_chunk,
+                   "parallelism": f"sequence-sharded x{world} (rank r owns global sequences {Bn}r..{Bn}r+{Bn - 1})",
                    "l2": "inputs larger than L2 (paged pool %.1f GiB)" % (cache.k.numel() * 4 / 2 ** 30)},
         "compaction_gbs": ach,
         "rows_moved_per_step": rows_moved / args.steps,
         "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
                                 "compact": t_compact / args.steps},
         "compact_ms_min_median_max": [per_compact[0], per_compact[len(per_compact) // 2], per_compact[-1]],
-        "step_hbm_gbs": (compact_bytes + score_bytes) / (ms / 1e3) / 1e9,
+        "step_hbm_gbs": (compact_bytes + score_bytes) / (ms / 1e3) / 1e9 if world == 1 else None,
         "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                      "frac": ach / peak, "peak_source": peak_src,
+                     "timed": "the compaction phase of every timed step (CUDA events on the launch stream around "
+                              "compact_stash_kernel + compact_kernel + compact_consumed_kernel)",
                      "traffic": traffic, "algorithmic_bytes_per_launch": compact_bytes / args.steps},
+        "kernels": kernels,
+        "kernels_note": f"per-kernel CUDA events over {kc_steps} further steps, each kernel bracketed by events "
+                        "(which also stops the early launch of the next kernel)",
         "gpu_launches": 6 * args.steps,   # Lag-KV partial, finalize, select, stash, compaction, eviction consumed
         "clocks": clk,
         "e2e": e2e,
     }
-    if world == 1 and not args.no_cpu_baseline and workload == WORKLOAD:
-        line["cpu_baseline"] = cpu_baseline()
-    print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+    return line
 
 
-def run_bandz2k(args):
-    """One step = a fresh sequence: its 2,048 tokens scored with the band-z
-    score (15 band layers of 4096 bf16), the cache cut to K = 512, all 32
-    layers' K/V compacted -- epikv_step on one sequence.  Each step's
-    sequence has its own resident cache and hidden rows."""
+# --------------------------------------------------------------------------- configuration 1
+def run_bandz2k(args, steps=None, warmup=None):
+    """Configuration 1.  One step = a fresh sequence: its 2,048 tokens scored
+    with the band-z score (15 band layers of 4096 bf16), the cache cut to
+    K = 512, all 32 layers' K/V compacted -- epikv_step on one sequence.
+    Each step's sequence has its own resident cache and hidden rows."""
     import torch
 
-    from paper_2606_26472_gb300 import build as B
     from paper_2606_26472_gb300 import epikv as E
     from paper_2606_26472_gb300.cache import KVCache
     from synth import workloads as W
     from synth.device import DeviceTrace
 
-    rank, local_rank, world = dist_env()
+    _, local_rank, world = dist_env()
     assert world == 1, "the band-z workload is a single-GPU measurement"
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if not os.path.exists(E.LIB_PATH):
-        B.build()
-    E.load()
+    dev = gpu_device(local_rank)
+    steps = args.steps if steps is None else steps
+    warmup = args.warmup if warmup is None else warmup
+    kc_steps = 3
     wl = W.config(1)
     m = wl.model
     T, K = wl.max_len, wl.budgets[0]
-    S = args.warmup + args.steps
+    S = warmup + steps + kc_steps
     nb = len(m.band_layers)
     dt = DeviceTrace(m, dev)
     cache = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, m.num_layers, m.num_kv_heads, m.head_dim, max_seqs=S, max_tokens=T,
@@ -537,30 +702,33 @@ def run_bandz2k(args):
     trigger = torch.tensor([K], dtype=torch.int32, device=dev)
     n_out = torch.empty(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
+    for s_ in range(S):
+        E.epikv_seq_reset(ctx, s_, 0, E.EPIKV_SCORE_BANDZ)
 
     def step(s_):
-        E.epikv_seq_reset(ctx, s_, 0, E.EPIKV_SCORE_BANDZ)
         E.epikv_step(ctx, 1, ids[s_], cu, T, budget, trigger, views[s_], kv, n_out)
 
-    for s_ in range(args.warmup):
+    for s_ in range(warmup):
         step(s_)
     torch.cuda.synchronize()
     stats0 = E.epikv_get_stats(ctx)
     phase = []
-    for _ in range(args.steps):
+    for _ in range(steps):
         evs = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         for e in evs:
             e.record(stream)
         phase.append(evs)
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(Clocks.device_id(dev, local_rank)).start()
     torch.cuda.synchronize()
     t0.record(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         E.epikv_set_phase_events(ctx, phase[i])
-        step(args.warmup + i)
+        step(warmup + i)
     t1.record(stream)
     torch.cuda.synchronize()
+    clk = clocks.stop()
     E.epikv_set_phase_events(ctx, None)
     ms = t0.elapsed_time(t1)
     stats1 = E.epikv_get_stats(ctx)
@@ -568,53 +736,60 @@ def run_bandz2k(args):
     assert st_ == E.EPIKV_OK, f"device error {code}"
     tokens = stats1["tokens_scored"] - stats0["tokens_scored"]
     rows = stats1["rows_moved"] - stats0["rows_moved"]
-    t_score = sum(p[0].elapsed_time(p[1]) for p in phase) / args.steps
-    t_select = sum(p[1].elapsed_time(p[2]) for p in phase) / args.steps
-    t_compact = sum(p[2].elapsed_time(p[3]) for p in phase) / args.steps
-    score_bytes = T * nb * m.hidden * 2 + 2 * nb * m.hidden * 2       # rows + h_prev write/read
-    compact_bytes = 2 * rows / args.steps * m.num_layers * 2 * m.num_kv_heads * m.head_dim * 2
+    t_score = sum(p[0].elapsed_time(p[1]) for p in phase) / steps
+    t_select = sum(p[1].elapsed_time(p[2]) for p in phase) / steps
+    t_compact = sum(p[2].elapsed_time(p[3]) for p in phase) / steps
+    sb = stream_bytes(m, tokens=T, seq_calls=1, rows_moved=rows / steps, kinds=E.EPIKV_SCORE_BANDZ, one_token=False)
+    score_bytes, compact_bytes = sb["bandz_g_kernel"], sb["compact_kernel"]
     peak, peak_src = measured_hbm_peak()
     g = score_bytes / (t_score / 1e3) / 1e9
     c = compact_bytes / (t_compact / 1e3) / 1e9
-    line = {"metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+    s_k0 = E.epikv_get_stats(ctx)
+    recs = kernel_pass(E, ctx, 8 * kc_steps, lambda: [step(warmup + steps + j) for j in range(kc_steps)])
+    s_k1 = E.epikv_get_stats(ctx)
+    kernels = kernel_table(recs, kc_steps, stream_bytes(m, tokens=T * kc_steps, seq_calls=kc_steps,
+                                                        rows_moved=s_k1["rows_moved"] - s_k0["rows_moved"],
+                                                        kinds=E.EPIKV_SCORE_BANDZ, one_token=False), peak)
+    E.epikv_destroy(ctx)
+    return {"metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1, "steps": steps,
+            "warmup": warmup, "ms_per_step": ms / steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": "single_2k_bandz_K512_fresh_sequence_per_step", "band_layers": nb,
                        "hidden": m.hidden, "budget_K": K, "layout": "contiguous",
+                       "step": "one fresh sequence: 2,048 tokens scored, one eviction 2,048 -> 512",
                        "l2": "inputs larger than L2 (%.1f GiB resident)" % ((cache.k.numel() * 2 + hid.numel()) * 2 / 2 ** 30)},
             "kernels_ms_per_step": {"score": t_score, "select": t_select, "compact": t_compact},
-            "score_phase_gbs": g, "compaction_gbs": c,
+            "score_phase_gbs": g, "compaction_gbs": c, "compaction_frac": c / peak,
             "roofline": {"bound": "hbm", "kernel": "score phase (bandz_g_kernel + score_finalize_kernel)",
                          "achieved": g, "peak": peak, "unit": "GB/s", "frac": g / peak, "peak_source": peak_src,
                          "traffic": None, "algorithmic_bytes_per_launch": score_bytes},
-            "gpu_launches": 7 * args.steps}   # reset, g, finalize, select, stash, compaction, eviction consumed
-    print(json.dumps(line), flush=True)
+            "kernels": kernels,
+            "gpu_launches": 6 * steps,   # g, finalize, select, stash, compaction, eviction consumed
+            "clocks": clk}
 
 
-def run_pertoken(args):
-    """The per-token regime of the 65,536-token band-z workload: 4 sequences,
-    one new token each per decode step, 15 band rows per token.  One bench
-    step = 64 decode steps, issued either call by call or as one CUDA graph
-    of 64 epikv_score_update calls (the per-step kernels are tiny, so launch
+# --------------------------------------------------------------------------- configuration 4
+def run_pertoken(args, steps=None, warmup=None):
+    """Configuration 4's per-token phase: 4 sequences, one new token each per
+    decode step, 15 band rows per token.  One bench step = 64 decode steps,
+    issued either call by call or as one CUDA graph of 64
+    epikv_score_update calls (the per-step kernels are tiny, so launch
     overhead decides the rate)."""
     import torch
 
-    from paper_2606_26472_gb300 import build as B
     from paper_2606_26472_gb300 import epikv as E
     from synth import workloads as W
     from synth.device import DeviceTrace
 
-    rank, local_rank, world = dist_env()
+    _, local_rank, world = dist_env()
     assert world == 1, "the per-token workload is a single-GPU measurement"
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if not os.path.exists(E.LIB_PATH):
-        B.build()
-    E.load()
+    dev = gpu_device(local_rank)
+    steps = args.steps if steps is None else steps
+    warmup = args.warmup if warmup is None else warmup
     wl = W.config(4)
     m = wl.model
     Bn, G = wl.n_seq, 64
-    n_tok = (2 * (args.warmup + args.steps) + 1) * G     # eager run, then graph run
+    n_tok = (2 * (warmup + steps) + 2) * G     # eager run, graph run, the per-kernel block
     nb = len(m.band_layers)
     dt = DeviceTrace(m, dev)
     hid = torch.empty((nb, n_tok, Bn, m.hidden), dtype=torch.bfloat16, device=dev)
@@ -651,41 +826,156 @@ def run_pertoken(args):
             E.epikv_score_update(ctx, Bn, seq_ids, cu, 1, views[t0 + k], kv_unused)
 
     def timed(run_block, t0):
-        for w in range(args.warmup):
+        for w in range(warmup):
             run_block(t0 + w * G)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for i in range(args.steps):
-            run_block(t0 + (args.warmup + i) * G)
+        for i in range(steps):
+            run_block(t0 + (warmup + i) * G)
         e1.record(stream)
         torch.cuda.synchronize()
         return e0.elapsed_time(e1)
 
     ms_eager = timed(eager_block, t)
-    t += (args.warmup + args.steps) * G
+    t += (warmup + steps) * G
     graphs = {}
-    for blk in range(args.warmup + args.steps):     # one graph per 64-token block, captured before timing
+    for blk in range(warmup + steps):     # one graph per 64-token block, captured before timing
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
             eager_block(t + blk * G)
         graphs[t + blk * G] = g
+    clocks = Clocks(Clocks.device_id(dev, local_rank)).start()
     ms_graph = timed(lambda t0: graphs[t0].replay(), t)
+    clk = clocks.stop()
+    t += (warmup + steps) * G
+    peak, _ = measured_hbm_peak()
+    recs = kernel_pass(E, ctx, G, lambda: eager_block(t))
+    kernels = kernel_table(recs, 1, stream_bytes(m, tokens=G * Bn, seq_calls=G * Bn, rows_moved=0,
+                                                 kinds=E.EPIKV_SCORE_BANDZ, one_token=True), peak)
     st_, code = E.epikv_get_error(ctx)
     assert st_ == E.EPIKV_OK, f"device error {code}"
-    tokens = args.steps * G * Bn
-    line = {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_graph / args.steps, "higher_is_better": True,
+    E.epikv_destroy(ctx)
+    tokens = steps * G * Bn
+    return {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1, "steps": steps,
+            "warmup": warmup, "ms_per_step": ms_graph / steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": "batch4_bandz_per_token_updates", "sequences": Bn, "band_layers": nb,
-                       "hidden": m.hidden, "step": "64 decode tokens per sequence",
+                       "hidden": m.hidden, "step": "64 decode tokens per sequence (one CUDA graph of 64 calls)",
                        "l2": "band rows of every token resident, %.1f GiB" % (hid.numel() * 2 / 2 ** 30)},
-            "per_token_us": {"graph": 1e3 * ms_graph / (args.steps * G), "eager": 1e3 * ms_eager / (args.steps * G)},
+            "per_token_us": {"graph": 1e3 * ms_graph / (steps * G), "eager": 1e3 * ms_eager / (steps * G)},
             "eager_value": tokens / (ms_eager / 1e3),
-            "gpu_launches": G * args.steps}   # one fused g + z launch per decode step
-    print(json.dumps(line), flush=True)
+            "kernels": kernels,
+            "gpu_launches": G * steps,   # one fused g + z launch per decode step
+            "clocks": clk}
 
 
+def run_evict64k(args, steps=None, warmup=None):
+    """Configuration 4's eviction phase: 4 sequences of 65,536 scored tokens
+    (band-z), each cut to K = 4,096 at once -- the radix select over 65,408
+    candidates per sequence (keys not staged in shared memory) and the
+    compaction of every layer's K and V.  Each timed eviction starts from the
+    same state: the workspace and the caches are restored (untimed) from a
+    device snapshot taken after scoring."""
+    import torch
+
+    from paper_2606_26472_gb300 import epikv as E
+    from paper_2606_26472_gb300.cache import KVCache
+    from synth import workloads as W
+    from synth.device import DeviceTrace
+
+    _, local_rank, world = dist_env()
+    assert world == 1, "the eviction workload is a single-GPU measurement"
+    dev = gpu_device(local_rank)
+    steps = min(args.steps, 5) if steps is None else steps
+    warmup = min(args.warmup, 2) if warmup is None else warmup
+    wl = W.config(4)
+    m = wl.model
+    Bn, T, K = wl.n_seq, wl.max_len, wl.budgets[0]
+    L, H, d, nb = m.num_layers, m.num_kv_heads, m.head_dim, len(m.band_layers)
+    CH = 4096                                       # tokens per scoring call (chunking does not change scores)
+    dt = DeviceTrace(m, dev)
+    cache = KVCache(E.EPIKV_LAYOUT_CONTIGUOUS, L, H, d, max_seqs=Bn, max_tokens=T, device=dev)
+    for b in range(Bn):
+        dt.kv(b, 0, T, 0, cache.k, cache.v, **cache.synth_kwargs())
+    cfg = E.make_config(max_seqs=Bn, max_cache_tokens=T, max_new_tokens=CH, n_band_a=len(m.band_a),
+                        n_band_b=len(m.band_b), score_kinds=E.EPIKV_SCORE_BANDZ)
+    ws = torch.empty(E.epikv_workspace_bytes(cfg), dtype=torch.uint8, device=dev)
+    ctx = E.epikv_init(cfg, ws, ws.numel())
+    for b in range(Bn):
+        E.epikv_seq_reset(ctx, b, 0, E.EPIKV_SCORE_BANDZ)
+    kv = cache.view()
+    hid = torch.empty((nb, Bn * CH, m.hidden), dtype=torch.bfloat16, device=dev)
+    hv = E.hidden_view([hid[i] for i in range(nb)], m.hidden)
+    seq_ids = torch.arange(Bn, dtype=torch.int32, device=dev)
+    cu = (torch.arange(Bn + 1, dtype=torch.int32, device=dev) * CH).contiguous()
+    for p0 in range(0, T, CH):
+        for b in range(Bn):
+            for i, layer in enumerate(m.band_layers):
+                dt.hidden(b, layer, p0, CH, hid[i, b * CH:(b + 1) * CH], m.hidden)
+        E.epikv_score_update(ctx, Bn, seq_ids, cu, CH, hv, kv)
+    del hid
+    torch.cuda.synchronize()
+    snap = (ws.clone(), cache.k.clone(), cache.v.clone())
+    kept = torch.empty((Bn, K), dtype=torch.int32, device=dev)
+    nk = torch.empty(Bn, dtype=torch.int32, device=dev)
+    bud = torch.full((Bn,), K, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def restore():
+        ws.copy_(snap[0])
+        cache.k.copy_(snap[1])
+        cache.v.copy_(snap[2])
+        torch.cuda.synchronize()
+
+    def evict():
+        E.epikv_select(ctx, Bn, seq_ids, bud, None, kept, K, nk)
+        E.epikv_compact(ctx, Bn, seq_ids, kept, K, kv)
+
+    for _ in range(warmup):
+        restore()
+        evict()
+    sel, cmp_, tot, rows = [], [], [], 0
+    clocks = Clocks(Clocks.device_id(dev, local_rank)).start()
+    for _ in range(steps):
+        restore()
+        s0 = E.epikv_get_stats(ctx)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        ev[0].record(stream)
+        E.epikv_select(ctx, Bn, seq_ids, bud, None, kept, K, nk)
+        ev[1].record(stream)
+        E.epikv_compact(ctx, Bn, seq_ids, kept, K, kv)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        rows += E.epikv_get_stats(ctx)["rows_moved"] - s0["rows_moved"]
+        sel.append(ev[0].elapsed_time(ev[1]))
+        cmp_.append(ev[1].elapsed_time(ev[2]))
+        tot.append(ev[0].elapsed_time(ev[2]))
+    clk = clocks.stop()
+    assert (nk.cpu().numpy() == K).all()
+    peak, peak_src = measured_hbm_peak()
+    restore()
+    s0 = E.epikv_get_stats(ctx)
+    recs = kernel_pass(E, ctx, 8, evict)
+    s1 = E.epikv_get_stats(ctx)
+    kernels = kernel_table(recs, 1, stream_bytes(m, tokens=0, seq_calls=0, rows_moved=s1["rows_moved"] - s0["rows_moved"],
+                                                 kinds=E.EPIKV_SCORE_BANDZ, one_token=False), peak)
+    st_, code = E.epikv_get_error(ctx)
+    assert st_ == E.EPIKV_OK, f"device error {code}"
+    E.epikv_destroy(ctx)
+    row_bytes = L * 2 * H * d * 2
+    cbytes = 2 * rows / steps * row_bytes
+    c_ms = float(np.median(cmp_))
+    return {"workload": "batch4_64k_bandz_single_eviction_to_K4096", "steps": steps, "warmup": warmup,
+            "ms_per_eviction": float(np.median(tot)), "select_ms": float(np.median(sel)), "compact_ms": c_ms,
+            "candidates_per_sequence": T - 128, "rows_moved_per_eviction": rows / steps,
+            "compaction_gbs": cbytes / (c_ms / 1e3) / 1e9, "compaction_frac": cbytes / (c_ms / 1e3) / 1e9 / peak,
+            "peak_source": peak_src, "kernels": kernels, "clocks": clk,
+            "timing": "median over evictions, each from the restored post-scoring state; CUDA events around "
+                      "epikv_select and epikv_compact"}
+
+
+# --------------------------------------------------------------------------- per-layer budgets
 def run_layers32k(args):
     """Per-layer budgets on the 32 x 32k Lag-KV paged workload: layer l of
     every sequence keeps its own budget K_l (a pyramid from 1.5 K at layer 0
@@ -701,19 +991,14 @@ def run_layers32k(args):
     stream).  The caches are filled by the same steps, untimed."""
     import torch
 
-    from paper_2606_26472_gb300 import build as B
     from paper_2606_26472_gb300 import epikv as E
     from paper_2606_26472_gb300.cache import KVCache
     from synth import gen, workloads as W
     from synth.device import DeviceTrace
 
-    rank, local_rank, world = dist_env()
+    _, local_rank, world = dist_env()
     assert world == 1, "the per-layer budget workload is a single-GPU measurement"
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if not os.path.exists(E.LIB_PATH):
-        B.build()
-    E.load()
+    dev = gpu_device(local_rank)
     wl = W.config(3)
     m = wl.model
     Bn, K, C = args.sequences, args.budget, args.chunk
@@ -778,8 +1063,7 @@ def run_layers32k(args):
         if st == t0:
             torch.cuda.synchronize()
             stats0 = E.epikv_get_stats(ctx)
-            clocks = Clocks(gpu_id)
-            clocks.start()
+            clocks = Clocks(gpu_id).start()
         write_new(st * C)
         E.epikv_set_phase_events(ctx, phase[st])
         ev[st][0].record(stream)
@@ -806,7 +1090,8 @@ def run_layers32k(args):
     peak, peak_src = measured_hbm_peak()
     ach = compact_bytes / (t_compact / 1e3) / 1e9
     block_bytes = 2 * bs * H * d * 2                        # K and V of one block
-    line = {
+    E.epikv_destroy(ctx)
+    return {
         "metric": METRIC, "value": tokens / (ms / 1e3), "unit": UNIT, "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
@@ -827,9 +1112,9 @@ def run_layers32k(args):
         "gpu_launches": (7 if Bn * L <= 256 else 6) * args.steps,
         "clocks": clk,
     }
-    print(json.dumps(line), flush=True)
 
 
+# --------------------------------------------------------------------------- configurations 2 and 5
 def window_schedule(n0, budgets, slack, C, n_calls):
     """The decode window's rows, simulated on the host: per call, every
     sequence's C new tokens (positions continuing from n0, slots from its
@@ -853,38 +1138,37 @@ def window_schedule(n0, budgets, slack, C, n_calls):
     return pos_tab, slot_tab, evict_tab, n_cache
 
 
-def run_window(args):
+def run_window(args, workload=None, steps=None, warmup=None):
     """Steady-state decode windows of two more workloads, timed per
     epikv_step call with CUDA events on the stream; the generator kernels
     that append each call's new rows (the model's side of the loop) run
     between the events:
-    * bandz8k: 8 x 8,192-token band-z traces, contiguous K/V, K = 4,096;
-      64 new tokens per sequence per call, every call evicts back to K;
-    * ragged64: 64 sequences with budgets from {2048, 4096, 8192}, paged
-      16-token blocks, both scores, one new token per sequence per call; a
-      sequence evicts when its cache exceeds K + 64.  The sequences start at
-      staggered lengths K + (29 b mod 65), so one of them evicts at nearly
-      every call.
+    * bandz8k (configuration 2): 8 x 8,192-token band-z traces, contiguous
+      K/V, K = 4,096; 64 new tokens per sequence per call, every call evicts
+      back to K;
+    * ragged64 (configuration 5): 64 sequences with budgets from {2048,
+      4096, 8192}, paged 16-token blocks, both scores, one new token per
+      sequence per call; a sequence evicts when its cache exceeds K + 64.
+      The sequences start at staggered lengths K + (29 b mod 65), so one of
+      them evicts at nearly every call.
     One bench step = the calls in which every sequence evicts once (1 and
     65).  Every call has the same arguments, so one captured CUDA graph of
     the call is replayed; the eager rate (with the per-phase breakdown) is
     reported beside it."""
     import torch
 
-    from paper_2606_26472_gb300 import build as B
     from paper_2606_26472_gb300 import epikv as E
     from paper_2606_26472_gb300.cache import KVCache
     from synth import gen, workloads as W
     from synth.device import DeviceBatchTrace
 
-    rank, local_rank, world = dist_env()
+    _, local_rank, world = dist_env()
     assert world == 1, "the decode-window workloads are single-GPU measurements"
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if not os.path.exists(E.LIB_PATH):
-        B.build()
-    E.load()
-    ragged = args.workload == "ragged64"
+    dev = gpu_device(local_rank)
+    workload = workload or args.workload
+    steps = args.steps if steps is None else steps
+    warmup = args.warmup if warmup is None else warmup
+    ragged = workload == "ragged64"
     wl = W.config(5 if ragged else 2)
     m = wl.model
     L, H, d, nb = m.num_layers, m.num_kv_heads, m.head_dim, len(m.band_layers)
@@ -898,7 +1182,8 @@ def run_window(args):
     phase0 = (np.arange(Bn) * 29) % cycle if C == 1 else np.zeros(Bn, np.int64)
     n0 = budgets + phase0
     T_cap = int(budgets.max()) + cycle
-    n_calls = 2 * (args.warmup + args.steps) * calls      # eager run, then graph run
+    kc_calls = calls if ragged else 3   # the per-kernel pass: one step of 65 calls, or 3 calls
+    n_calls = 2 * (warmup + steps) * calls + kc_calls     # eager run, graph run, per-kernel pass
     max_pos = int(n0.max()) + n_calls * C + 1
     paged = wl.layout == W.PAGED
     if paged:
@@ -991,79 +1276,163 @@ def run_window(args):
         return ms, per_phase
 
     gpu_id = Clocks.device_id(dev, local_rank)
-    window(args.warmup, call, False)
+    window(warmup, call, False)
     s0 = E.epikv_get_stats(ctx)
     j0 = j
-    ms_eager, (t_score, t_select, t_compact) = window(args.steps, call, True, phases=True)
+    ms_eager, (t_score, t_select, t_compact) = window(steps, call, True, phases=True)
     s1 = E.epikv_get_stats(ctx)
     assert s1["evictions"] - s0["evictions"] == int(evict_tab[j0:j].sum())
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
         call()
-    window(args.warmup, g.replay, False)
-    clocks = Clocks(gpu_id)
-    clocks.start()
+    window(warmup, g.replay, False)
+    clocks = Clocks(gpu_id).start()
     s2 = E.epikv_get_stats(ctx)
     j2 = j
-    ms_graph, _ = window(args.steps, g.replay, True)
+    ms_graph, _ = window(steps, g.replay, True)
     clk = clocks.stop()
     s3 = E.epikv_get_stats(ctx)
-    assert j == n_calls
     assert s3["evictions"] - s2["evictions"] == int(evict_tab[j2:j].sum())
+    # per-kernel CUDA events over kc_calls eager calls
+    peak, peak_src = measured_hbm_peak()
+
+    def kc_run():
+        nonlocal j
+        for _ in range(kc_calls):
+            append(j)
+            call()
+            j += 1
+
+    s4 = E.epikv_get_stats(ctx)
+    recs = kernel_pass(E, ctx, 8 * kc_calls, kc_run)
+    s5 = E.epikv_get_stats(ctx)
+    assert j == n_calls
+    kernels = kernel_table(recs, kc_calls / calls,
+                           stream_bytes(m, tokens=kc_calls * Bn * C, seq_calls=kc_calls * Bn,
+                                        rows_moved=s5["rows_moved"] - s4["rows_moved"], kinds=wl.kinds,
+                                        one_token=C == 1), peak)
     st_, code = E.epikv_get_error(ctx)
     assert st_ == E.EPIKV_OK, f"device error {code}"
     for b in range(Bn):   # the device's cache lengths follow the host's simulation
         _, _, n = E.epikv_read_slots(ctx, b, wl.policies[b], 1)
         assert n == n_cache[b], (b, n, int(n_cache[b]))
+    E.epikv_destroy(ctx)
 
-    tokens = args.steps * calls * Bn * C
+    tokens = steps * calls * Bn * C
     assert s3["tokens_scored"] - s2["tokens_scored"] == tokens
     row_bytes = L * 2 * H * d * 2
     rows = s1["rows_moved"] - s0["rows_moved"]
     compact_bytes = 2 * rows * row_bytes
-    n_launch = calls * args.steps
-    peak, peak_src = measured_hbm_peak()
+    n_launch = calls * steps
     ach = compact_bytes / (t_compact / 1e3) / 1e9
-    workload = ("ragged64_4k32k_both_paged16_steady" if ragged else "batch8_8k_bandz_contiguous_K4096_every64")
-    line = {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_graph / args.steps,
+    name = ("ragged64_4k32k_both_paged16_steady" if ragged else "batch8_8k_bandz_contiguous_K4096_every64")
+    return {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1,
+            "steps": steps, "warmup": warmup, "ms_per_step": ms_graph / steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": workload, "sequences": Bn, "budgets": sorted(set(wl.budgets)),
+            "config": {"workload": name, "sequences": Bn, "budgets": sorted(set(wl.budgets)),
                        "new_tokens_per_call": C, "calls_per_step": calls,
                        "evict_when": f"n_cache > K + {slack}", "layout": "paged16_shuffled" if paged else "contiguous",
                        "score_kinds": wl.kinds, "timing": "CUDA events around each epikv_step call, queued behind a device spin",
                        "l2": "K/V caches %.1f GiB, larger than L2" % (cache.k.numel() * 4 / 2 ** 30)},
             "eager_value": tokens / (ms_eager / 1e3),
             "us_per_call": {"graph": 1e3 * ms_graph / n_launch, "eager": 1e3 * ms_eager / n_launch},
-            "kernels_ms_per_step": {"score": t_score / args.steps, "select": t_select / args.steps,
-                                    "compact": t_compact / args.steps},
-            "evictions_per_step": (s1["evictions"] - s0["evictions"]) / args.steps,
-            "compaction_gbs": ach,
+            "kernels_ms_per_step": {"score": t_score / steps, "select": t_select / steps,
+                                    "compact": t_compact / steps},
+            "evictions_per_step": (s1["evictions"] - s0["evictions"]) / steps,
+            "compaction_gbs": ach, "compaction_frac": ach / peak,
             "roofline": {"bound": "hbm", "kernel": "compact_kernel", "achieved": ach, "peak": peak, "unit": "GB/s",
                          "frac": ach / peak, "peak_source": peak_src, "traffic": None,
                          "algorithmic_bytes_per_launch": compact_bytes / n_launch,
                          "timing": "eager calls, phase events"},
+            "kernels": kernels,
             # one-token calls: the fused score kernel, select, stash, compaction, eviction
             # consumed; longer calls: g, [Lag-KV partial,] finalize and the same four
             "gpu_launches": (5 if C == 1 else (7 if wl.kinds & E.EPIKV_SCORE_LAGKV else 6)) * n_launch,
             "clocks": clk}
-    print(json.dumps(line), flush=True)
 
 
-def main():
-    args = parse()
+# --------------------------------------------------------------------------- the per-configuration table
+def _entry(res, step):
+    keys = ("value", "unit", "ms_per_step", "steps", "warmup", "compaction_gbs", "compaction_frac",
+            "kernels_ms_per_step", "kernels", "clocks")
+    out = {"workload": res["config"]["workload"], "step": step}
+    out.update({k: res[k] for k in keys if k in res})
+    return out
+
+
+def collect_configs(args, headline):
+    """Every workload measured one after another on this GPU (each with its
+    own clocks record and per-kernel CUDA-event pass), reduced step counts."""
+    import gc
+
+    import torch
+
+    def free():
+        gc.collect()
+        torch.cuda.empty_cache()
+
+    t0 = time.time()
+    out = {}
+    free()
+    r = run_bandz2k(args, steps=10, warmup=3)
+    out["1"] = _entry(r, "one fresh sequence: 2,048 tokens scored (band-z), one eviction 2,048 -> 512")
+    out["1"]["score_phase_gbs"] = r["score_phase_gbs"]
+    free()
+    r = run_window(args, "bandz8k", steps=20, warmup=3)
+    out["2"] = _entry(r, "one epikv_step call (CUDA graph): 64 new tokens of each of 8 sequences scored (band-z), "
+                         "every cache 4,160 -> 4,096")
+    out["2"]["eager_value"] = r["eager_value"]
+    h = headline
+    out["3"] = {"workload": h["config"]["workload"], "step": "one epikv_step: 128 new tokens of each of 32 "
+                "sequences scored (Lag-KV), every cache 8,320 -> 8,192", "value": h["value"], "unit": h["unit"],
+                "ms_per_step": h["ms_per_step"], "steps": h["steps"], "warmup": h["warmup"],
+                "compaction_gbs": h["compaction_gbs"], "compaction_frac": h["roofline"]["frac"],
+                "kernels_ms_per_step": h["kernels_ms_per_step"], "kernels": h["kernels"], "clocks": h["clocks"],
+                "note": "the headline measurement of this line"}
+    free()
+    r4a = run_pertoken(args, steps=10, warmup=3)
+    free()
+    r4b = run_evict64k(args, steps=3, warmup=1)
+    free()
+    per_step_ms = r4a["ms_per_step"] / 64          # one decode step of the 4 sequences (graph replay)
+    whole_ms = 65536 * per_step_ms + r4b["ms_per_eviction"]
+    out["4"] = {"workload": "batch4_64k_bandz_K4096", "step": "per-token phase: 64 decode steps of 4 sequences "
+                "(one CUDA graph of 64 score updates); eviction phase: 4 x 65,536 -> 4,096",
+                "per_token_phase": _entry(r4a, "64 decode steps (4 tokens each)"),
+                "eviction_phase": r4b,
+                "whole_schedule_tokens_per_s": 4 * 65536 / (whole_ms / 1e3),
+                "whole_schedule_note": "4 x 65,536 tokens over 65,536 x the measured decode-step time plus the "
+                                       "measured eviction (the phases are measured apart)"}
+    r = run_window(args, "ragged64", steps=3, warmup=2)
+    free()
+    out["5"] = _entry(r, "65 epikv_step calls (CUDA graph), one new token of each of 64 sequences per call "
+                         "(both scores); every sequence evicts once")
+    out["5"]["us_per_call"] = r["us_per_call"]
+    out["5"]["eager_value"] = r["eager_value"]
+    out["seconds"] = time.time() - t0
+    return out
+
+
+def main(argv=None):
+    args = parse(argv)
     if args.impl == "reference":
         run_reference(args)
-    elif args.workload == "bandz2k":
-        run_bandz2k(args)
-    elif args.workload == "pertoken":
-        run_pertoken(args)
-    elif args.workload == "layers32k":
-        run_layers32k(args)
-    elif args.workload in ("bandz8k", "ragged64"):
-        run_window(args)
-    else:
-        run_ours(args)
+        return
+    if args.workload == "lagkv32k":
+        line = run_ours(args)
+        if line is None:
+            return
+        _, _, world = dist_env()
+        default = line["config"]["workload"] == WORKLOAD
+        if world == 1 and default and not args.no_configs:
+            line["configs"] = collect_configs(args, line)
+        if world == 1 and default and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(args.cpu_workers)
+        print(json.dumps(line), flush=True)
+        return
+    run = {"bandz2k": run_bandz2k, "pertoken": run_pertoken, "evict64k": run_evict64k, "layers32k": run_layers32k,
+           "bandz8k": run_window, "ragged64": run_window}[args.workload]
+    print(json.dumps(run(args)), flush=True)
 
 
 if __name__ == "__main__":

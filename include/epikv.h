@@ -265,6 +265,21 @@ epikv_status epikv_step(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
  * NULL stops it.  The events are the caller's. */
 epikv_status epikv_set_phase_events(epikv_ctx* ctx, const cudaEvent_t* events);
 
+/* Per-kernel timing for measurement.  From this call on, every kernel that an
+ * entry point of `ctx` launches (epikv_score_update, epikv_select,
+ * epikv_compact, epikv_step) is bracketed on its stream by two of the
+ * caller's events -- events[2k] before and events[2k+1] after the k-th such
+ * kernel -- and h_names[k] receives its name as the CUDA runtime reports it
+ * (storage owned by the runtime), for at most n_kernels kernels; later ones
+ * are not recorded.  Both arrays are the caller's and must stay valid until
+ * the next call.  An event recorded between two kernels also ends the early
+ * launch of the second (programmatic dependent launch), so the kernels then
+ * run strictly one after another.  events == NULL stops it and, if h_used is
+ * not NULL, stores how many kernels were recorded.  Not thread safe with
+ * respect to other calls on the same context. */
+epikv_status epikv_set_kernel_events(epikv_ctx* ctx, const cudaEvent_t* events, int32_t n_kernels,
+                                     const char** h_names, int32_t* h_used);
+
 /* Debug/test read-back (synchronises): the cache length, positions and
  * scores of kind `kind` of `seq`'s slots; at most `cap` entries copied. */
 epikv_status epikv_read_slots(epikv_ctx* ctx, int32_t seq, int32_t kind, float* h_score,

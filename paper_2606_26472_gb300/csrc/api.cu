@@ -21,6 +21,8 @@ struct epikv_ctx {
   cudaStream_t last_stream;
   bool timing;
   cudaEvent_t ev[4];
+  bool kclock_on;
+  KernelClock kclock;   // per-kernel events (epikv_set_kernel_events)
 };
 
 namespace {
@@ -180,6 +182,13 @@ bool valid_hidden(const epikv_ctx* ctx, const epikv_hidden_view* hv) {
 
 epikv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? EPIKV_OK : EPIKV_ECUDA; }
 
+// Points the launch helpers at the context's kernel events (if set) for the
+// duration of one entry point.
+struct ClockScope {
+  explicit ClockScope(epikv_ctx* ctx) { t_kernel_clock = ctx && ctx->kclock_on ? &ctx->kclock : nullptr; }
+  ~ClockScope() { t_kernel_clock = nullptr; }
+};
+
 }  // namespace
 
 extern "C" {
@@ -249,6 +258,7 @@ epikv_status epikv_score_update(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_
                                 int32_t max_new, const epikv_hidden_view* hidden, const epikv_kv_view* kv,
                                 cudaStream_t stream) {
   int launches = 0;
+  ClockScope clock(ctx);
   return score_update_impl(ctx, n_seq, d_seq_ids, d_cu_new, max_new, hidden, kv, stream, &launches);
 }
 
@@ -259,6 +269,7 @@ epikv_status epikv_select(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_id
   if (n_seq > 0 && (!d_seq_ids || !d_budget || !d_kept)) return EPIKV_EINVAL;
   ctx->last_stream = stream;
   int launches = 0;
+  ClockScope clock(ctx);
   return cuda_status(launch_select(ctx->st, ctx->dm, n_seq, d_seq_ids, d_budget, d_trigger, d_kept, kept_stride,
                                    d_n_kept, stream, &launches));
 }
@@ -271,6 +282,7 @@ epikv_status epikv_compact(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_i
   if (!valid_kv(ctx, kv, &kd)) return EPIKV_EINVAL;
   ctx->last_stream = stream;
   int launches = 0;
+  ClockScope clock(ctx);
   return cuda_status(
       launch_compact(ctx->st, ctx->dm, n_seq, d_seq_ids, d_kept, kept_stride, kd, ctx->compact_ctas, stream, &launches));
 }
@@ -285,6 +297,7 @@ epikv_status epikv_step(epikv_ctx* ctx, int32_t n_seq, const int32_t* d_seq_ids,
   KvDev kd;
   if (!valid_kv(ctx, kv, &kd)) return EPIKV_EINVAL;
   int launches = 0;
+  ClockScope clock(ctx);
   cudaError_t e = cudaSuccess;
   if (ctx->timing) e = cudaEventRecord(ctx->ev[0], stream);
   if (e != cudaSuccess) return EPIKV_ECUDA;
@@ -313,6 +326,27 @@ epikv_status epikv_set_phase_events(epikv_ctx* ctx, const cudaEvent_t* events) {
     ctx->ev[i] = events[i];
   }
   ctx->timing = true;
+  return EPIKV_OK;
+}
+
+epikv_status epikv_set_kernel_events(epikv_ctx* ctx, const cudaEvent_t* events, int32_t n_kernels,
+                                     const char** h_names, int32_t* h_used) {
+  if (!ctx) return EPIKV_EINVAL;
+  if (!events) {
+    if (h_used) *h_used = ctx->kclock_on ? ctx->kclock.used : 0;
+    ctx->kclock_on = false;
+    return EPIKV_OK;
+  }
+  if (n_kernels < 1 || !h_names) return EPIKV_EINVAL;
+  for (int i = 0; i < 2 * n_kernels; ++i)
+    if (!events[i]) return EPIKV_EINVAL;
+  for (int i = 0; i < n_kernels; ++i) h_names[i] = nullptr;
+  ctx->kclock.ev = const_cast<cudaEvent_t*>(events);
+  ctx->kclock.names = h_names;
+  ctx->kclock.cap = n_kernels;
+  ctx->kclock.used = 0;
+  ctx->kclock_on = true;
+  if (h_used) *h_used = 0;
   return EPIKV_OK;
 }
 

@@ -101,8 +101,8 @@ __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.lau
 #endif
 
 template <typename... Params, typename... Args>
-inline cudaError_t launch_kernel(bool programmatic, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
-                                 cudaStream_t stream, Args... args) {
+inline cudaError_t launch_kernel_now(bool programmatic, void (*kernel)(Params...), dim3 grid, dim3 block,
+                                     size_t smem, cudaStream_t stream, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -115,6 +115,36 @@ inline cudaError_t launch_kernel(bool programmatic, void (*kernel)(Params...), d
   cfg.numAttrs = programmatic && EPIKV_PDL ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
+
+// Per-kernel timing (epikv_set_kernel_events): while an entry point of a
+// context with kernel events runs, t_kernel_clock points at its record, and
+// every kernel it launches is bracketed by two of the caller's events on the
+// launch stream, its name (cudaFuncGetName) stored beside them.
+struct KernelClock {
+  cudaEvent_t* ev;      // [2 * cap]: before and after each kernel
+  const char** names;   // [cap]
+  int cap, used;
+};
+inline thread_local KernelClock* t_kernel_clock = nullptr;
+
+template <typename... Params, typename... Args>
+inline cudaError_t launch_kernel(bool programmatic, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                                 cudaStream_t stream, Args... args) {
+  KernelClock* kc = t_kernel_clock;
+  if (kc && kc->used < kc->cap) {
+    const cudaError_t e = cudaEventRecord(kc->ev[2 * kc->used], stream);
+    if (e != cudaSuccess) return e;
+  } else {
+    kc = nullptr;
+  }
+  const cudaError_t e = launch_kernel_now(programmatic, kernel, grid, block, smem, stream, args...);
+  if (e != cudaSuccess || !kc) return e;
+  const char* name = nullptr;
+  if (cudaFuncGetName(&name, reinterpret_cast<const void*>(kernel)) != cudaSuccess) name = nullptr;
+  kc->names[kc->used] = name;
+  return cudaEventRecord(kc->ev[2 * kc->used++ + 1], stream);
+}
+
 
 template <typename... Params, typename... Args>
 inline cudaError_t pdl_launch(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,

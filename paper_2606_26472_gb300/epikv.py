@@ -56,6 +56,7 @@ _SIGS = {
     "epikv_step": (C.c_int, [_P, _I, _P, _P, _I, _P, _P, C.POINTER(epikv_hidden_view),
                              C.POINTER(epikv_kv_view), _P, _P]),
     "epikv_set_phase_events": (C.c_int, [_P, _P]),
+    "epikv_set_kernel_events": (C.c_int, [_P, _P, _I, _P, C.POINTER(_I)]),
     "epikv_read_slots": (C.c_int, [_P, _I, _I, _P, _P, _I, C.POINTER(_I)]),
     "epikv_read_layer_slots": (C.c_int, [_P, _I, _I, _P, _I, C.POINTER(_I)]),
     "epikv_get_stats": (C.c_int, [_P, C.POINTER(epikv_stats)]),
@@ -183,6 +184,48 @@ def epikv_set_phase_events(ctx, events):
         return
     arr = (C.c_void_p * 4)(*[e.cuda_event for e in events])
     _check(load().epikv_set_phase_events(ctx, arr), "epikv_set_phase_events")
+
+
+class KernelClock:
+    """Per-kernel CUDA events of a context (epikv_set_kernel_events): every
+    kernel the context's calls launch is bracketed by two events on its
+    stream.  `start()` arms it, `stop()` returns [(kernel name, ms)] in launch
+    order (synchronising on the last event)."""
+
+    def __init__(self, ctx, cap):
+        import torch
+        self.ctx, self.cap = ctx, cap
+        self.events = [torch.cuda.Event(enable_timing=True) for _ in range(2 * cap)]
+        s = torch.cuda.current_stream()
+        for e in self.events:
+            e.record(s)            # materialise the handles
+        self._ev = (C.c_void_p * (2 * cap))(*[e.cuda_event for e in self.events])
+        self._names = (C.c_char_p * cap)()
+
+    def start(self):
+        _check(load().epikv_set_kernel_events(self.ctx, self._ev, self.cap, self._names, None),
+               "epikv_set_kernel_events")
+
+    def stop(self):
+        used = C.c_int32()
+        _check(load().epikv_set_kernel_events(self.ctx, None, 0, None, C.byref(used)), "epikv_set_kernel_events")
+        n = used.value
+        if n:
+            self.events[2 * n - 1].synchronize()
+        return [((self._names[k] or b"?").decode(), self.events[2 * k].elapsed_time(self.events[2 * k + 1]))
+                for k in range(n)]
+
+
+def kernel_short_name(name):
+    """'epikv::compact_kernel<true>' style names from the runtime's (possibly
+    mangled) kernel name: the function's identifier only."""
+    import re
+    for ident in ("bandz_g_kernel", "bandz_token_kernel", "lagkv_partial_kernel", "score_finalize_kernel",
+                  "token_kernel", "select_kernel", "layer_keep_kernel", "layer_union_kernel", "compact_stash_kernel",
+                  "compact_consumed_kernel", "compact_kernel"):
+        if re.search(r"(?<![A-Za-z_])" + ident, name):
+            return ident
+    return name
 
 
 def epikv_read_slots(ctx, seq, kind, cap):

@@ -3,6 +3,7 @@
 sequence per call but one, and never writes past a cache's capacity; the
 8 x 8k schedule evicts every sequence at every call."""
 import numpy as np
+import pytest
 
 import bench
 from synth import workloads as W
@@ -37,3 +38,26 @@ def test_bandz8k_schedule_evicts_every_call():
     assert (ev == wl.n_seq).all()
     assert (slots.reshape(5, wl.n_seq, C)[:, :, 0] == budgets[None, :]).all()   # new rows from slot K each call
     assert (n_end == budgets).all()
+
+
+def test_stream_bytes_and_kernel_table():
+    """The algorithmic byte counts the bench divides by kernel times, on the
+    32k workload's numbers, and the per-kernel table built from event records."""
+    import bench
+    from synth import workloads as W
+    m = W.config(3).model
+    row, state, band = 32 * 2 * 8 * 128 * 2, 32 * 2 * 4 * 8 * 128 * 2, 15 * 4096 * 2
+    b = bench.stream_bytes(m, tokens=32 * 128, seq_calls=32, rows_moved=1000, kinds=2, one_token=False)
+    assert b == {"compact_kernel": 2 * 1000 * row, "lagkv_partial_kernel": 32 * 128 * row + 32 * 2 * state}
+    b = bench.stream_bytes(m, tokens=64, seq_calls=64, rows_moved=0, kinds=3, one_token=True)
+    assert b["token_kernel"] == 64 * (3 * band + row + 2 * state)
+    b = bench.stream_bytes(m, tokens=4, seq_calls=4, rows_moved=0, kinds=1, one_token=True)
+    assert b["bandz_token_kernel"] == 4 * 3 * band and "token_kernel" not in b
+    b = bench.stream_bytes(m, tokens=2048, seq_calls=1, rows_moved=0, kinds=8, one_token=False)
+    assert b["lagkv_partial_kernel"] == 2048 * row              # raw variances keep no range state
+    recs = [("_ZN5epikv14compact_kernelILb0EEEvv", 2.0), ("_ZN5epikv13select_kernelILb0EEEvv", 0.5),
+            ("_ZN5epikv14compact_kernelILb0EEEvv", 4.0)]
+    t = bench.kernel_table(recs, 2, {"compact_kernel": 6e9}, 6000.0)
+    assert t["compact_kernel"]["launches_per_step"] == 1 and t["compact_kernel"]["ms_per_step"] == 3.0
+    assert t["compact_kernel"]["gbs"] == pytest.approx(1000.0) and t["compact_kernel"]["hbm_frac"] == pytest.approx(1 / 6)
+    assert "gbs" not in t["select_kernel"]
