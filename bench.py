@@ -78,6 +78,10 @@ def parse(argv=None):
     p.add_argument("--select-chunk", type=int, default=1)
     # oracle processes of the CPU baseline (0: one per available core)
     p.add_argument("--cpu-workers", type=int, default=0)
+    # a scaled-down variant of the decode-window workloads (bandz8k, ragged64)
+    # for profiler captures: their first N sequences, and one budget for all
+    p.add_argument("--window-seqs", type=int, default=0)
+    p.add_argument("--window-budget", type=int, default=0)
     return p.parse_args(argv)
 
 
@@ -1170,6 +1174,13 @@ def run_window(args, workload=None, steps=None, warmup=None):
     warmup = args.warmup if warmup is None else warmup
     ragged = workload == "ragged64"
     wl = W.config(5 if ragged else 2)
+    scaled = bool(args.window_seqs or args.window_budget)
+    if scaled:
+        import dataclasses
+        n_keep = args.window_seqs or wl.n_seq
+        bud = (args.window_budget,) * n_keep if args.window_budget else wl.budgets[:n_keep]
+        wl = dataclasses.replace(wl, n_seq=n_keep, lengths=wl.lengths[:n_keep], budgets=bud,
+                                 policies=wl.policies[:n_keep], trigger_slack=wl.trigger_slack[:n_keep])
     m = wl.model
     L, H, d, nb = m.num_layers, m.num_kv_heads, m.head_dim, len(m.band_layers)
     Bn, C = wl.n_seq, wl.chunk
@@ -1326,6 +1337,8 @@ def run_window(args, workload=None, steps=None, warmup=None):
     n_launch = calls * steps
     ach = compact_bytes / (t_compact / 1e3) / 1e9
     name = ("ragged64_4k32k_both_paged16_steady" if ragged else "batch8_8k_bandz_contiguous_K4096_every64")
+    if scaled:
+        name += f"_first{Bn}seqs" + (f"_K{args.window_budget}" if args.window_budget else "")
     return {"metric": METRIC, "value": tokens / (ms_graph / 1e3), "unit": UNIT, "n_gpus": 1,
             "steps": steps, "warmup": warmup, "ms_per_step": ms_graph / steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",

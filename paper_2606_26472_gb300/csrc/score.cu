@@ -16,6 +16,8 @@
 // and u values are computed from the same bytes in the same order whether the
 // previous row comes from the call or from the saved state, and the window
 // reductions run over positions in a fixed lane order.
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -199,10 +201,20 @@ __device__ __forceinline__ uint4 q_max(const uint4& a, const uint4& b) {
 typedef unsigned long long f32x2;
 
 __device__ __forceinline__ f32x2 f2_pack(float lo, float hi) {
-  return ((f32x2)__float_as_uint(hi) << 32) | (f32x2)__float_as_uint(lo);
+  f32x2 d;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
+  return d;
 }
-__device__ __forceinline__ float f2_lo(f32x2 v) { return __uint_as_float((uint32_t)v); }
-__device__ __forceinline__ float f2_hi(f32x2 v) { return __uint_as_float((uint32_t)(v >> 32)); }
+__device__ __forceinline__ float f2_lo(f32x2 v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return lo;
+}
+__device__ __forceinline__ float f2_hi(f32x2 v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return hi;
+}
 __device__ __forceinline__ f32x2 f2_fma(f32x2 a, f32x2 b, f32x2 c) {
   f32x2 d;
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
@@ -231,7 +243,7 @@ __device__ __forceinline__ void prev_affine(const uint4& pmn, const uint4& pmx, 
   unpack8(pmx, mx);
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
-    inv[e] = 1.f / (mx[e] - mn[e] + eps);
+    inv[e] = __frcp_rn(mx[e] - mn[e] + eps);   // the correctly rounded reciprocal (as 1.f / x)
     bias[e] = fmaf(-mn[e], inv[e], -0.5f);
   }
 #pragma unroll
@@ -301,7 +313,10 @@ __device__ __forceinline__ void transpose_sum(float (&v)[NV], int lane) {
 // sums are the same bit for bit).  With HALF, each half of a 256-thread
 // block runs its own stream (K in the first half, V in the second; H*d/8 <=
 // 128), with its own shared memory.
-template <int LH, int SEG = kLagSeg, bool HALF = false>
+// KINDS: 0 = whichever K/V kinds the context computes (runtime flags); 1 =
+// the normalised kinds only; 2 = the raw kinds only; 3 = both (compile-time,
+// so a kernel instance holds only the registers its kinds need).
+template <int LH, int SEG = kLagSeg, bool HALF = false, int KINDS = 0>
 __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, const KvDev& kv, int seq,
                                            int n_new, int layer, int kvk, int nc0) {
   const int stream = layer * 2 + kvk;  // this stream's column of the per-token partials
@@ -313,8 +328,8 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
   const int hd = dm.H * dm.d;
   const int p0 = st.n_seen[seq];
   const int ch = h * dm.d + q * 8;  // first channel of this thread within the token row
-  const bool need_norm = dm.kinds & kNormKinds;   // uniform across the grid
-  const bool need_raw = dm.kinds & kRawKinds;
+  const bool need_norm = KINDS ? (KINDS & 1) != 0 : (dm.kinds & kNormKinds) != 0;   // uniform across the grid
+  const bool need_raw = KINDS ? (KINDS & 2) != 0 : (dm.kinds & kRawKinds) != 0;
   __nv_bfloat16* rng = need_norm ? st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd : nullptr;
 
   uint4 pmn = make_uint4(0, 0, 0, 0), pmx = pmn, cmn = pmn, cmx = pmn;
@@ -329,6 +344,7 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
 
   const float inv_d = 1.f / (float)dm.d;
   const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
+  const char* kvb_ch = kvbase + (int64_t)ch * 2;       // this thread's first channel in a row at offset 0
   __shared__ int64_t soff_s[HALF ? 2 : 1][kLagOffs];
   constexpr int NV = 2 * SEG;      // moments of a segment: (sum y, sum y^2) per token
   __shared__ float red_s[HALF ? 2 : 1][2][32][NV];  // [half][segment parity][head][moment]; the host admits H <= 32
@@ -350,65 +366,70 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
       const int seg = min(min(dm.lag - r, gn - i), SEG);
       const bool has_prev = p0 + g0 + i >= dm.lag;   // the segment's chunk is not chunk 0
       uint4 x[SEG];
-#pragma unroll
-      for (int j = 0; j < SEG; ++j) {
-        x[j] = make_uint4(0, 0, 0, 0);
-        if (j < seg && active) {
-          const int64_t off = soff[i + j];
-          if (off >= 0)
-            x[j] = ld_stream16(kvbase + (off + ch) * 2);
-          else
-            set_error(st.err, EPIKV_DEV_SLOT);
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < SEG; ++j) {
-        if (j < seg) {
-          if (need_raw) {  // population variance of the stored vector over the head dimension
-            float xf[8], s1 = 0.f;
-            unpack8(x[j], xf);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) s1 += xf[e];
-            const float mean = group_sum(s1, LH) * inv_d;
-            float s2 = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float dv = xf[e] - mean;
-              s2 = fmaf(dv, dv, s2);
-            }
-            const float var_raw = group_sum(s2, LH) * inv_d;
-            if (q == 0 && active) hr[parity][j][h] = var_raw;
-          }
-        }
-      }
-      if (has_prev && need_norm) {  // uniform across the block
-        float v[NV];
+      // FULL: every token of the segment is taken (the common case), so the
+      // per-token conditions compile away; the arithmetic is the same
+      auto body = [&](auto full_t) {
+        constexpr bool FULL = decltype(full_t)::value;
+        bool bad = false;
 #pragma unroll
         for (int j = 0; j < SEG; ++j) {
-          v[2 * j] = v[2 * j + 1] = 0.f;
-          if (j < seg) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
+          const bool take = (FULL || j < seg) && active;
+          const int64_t off = take ? soff[i + j] : 0;
+          bad |= off < 0;
+          x[j] = ld_stream16_if(kvb_ch + off * 2, take && off >= 0);
         }
-        transpose_sum<LH / 2, NV, NV>(v, tid & 31);
-        if (active) {
-          if constexpr (LH <= NV) {
+        if (bad) set_error(st.err, EPIKV_DEV_SLOT);
+        if (need_raw) {  // population variance of the stored vector over the head dimension
 #pragma unroll
-            for (int k = 0; k < NV / LH; ++k) red[parity][h][k + (NV / LH) * q] = v[k];
-          } else {
-            if (q % (LH / NV) == 0) red[parity][h][q / (LH / NV)] = v[0];
+          for (int j = 0; j < SEG; ++j) {
+            if (FULL || j < seg) {
+              float xf[8], s1 = 0.f;
+              unpack8(x[j], xf);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) s1 += xf[e];
+              const float mean = group_sum(s1, LH) * inv_d;
+              float s2 = 0.f;
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                const float dv = xf[e] - mean;
+                s2 = fmaf(dv, dv, s2);
+              }
+              const float var_raw = group_sum(s2, LH) * inv_d;
+              if (q == 0 && active) hr[parity][j][h] = var_raw;
+            }
           }
         }
-      }
-      // advance the running range of the current chunk
-      if (r == 0) {
-        cmn = x[0];
-        cmx = x[0];
-      }
+        if (has_prev && need_norm) {  // uniform across the block
+          float v[NV];
 #pragma unroll
-      for (int j = 0; j < SEG; ++j)
-        if (j < seg) {
-          cmn = q_min(cmn, x[j]);
-          cmx = q_max(cmx, x[j]);
+          for (int j = 0; j < SEG; ++j) {
+            v[2 * j] = v[2 * j + 1] = 0.f;
+            if (FULL || j < seg) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
+          }
+          transpose_sum<LH / 2, NV, NV>(v, tid & 31);
+          if (active) {
+            if constexpr (LH <= NV) {
+#pragma unroll
+              for (int k = 0; k < NV / LH; ++k) red[parity][h][k + (NV / LH) * q] = v[k];
+            } else {
+              if (q % (LH / NV) == 0) red[parity][h][q / (LH / NV)] = v[0];
+            }
+          }
         }
+        // advance the running range of the current chunk
+        if (r == 0) {
+          cmn = x[0];
+          cmx = x[0];
+        }
+#pragma unroll
+        for (int j = 0; j < SEG; ++j)
+          if (FULL || j < seg) {
+            cmn = q_min(cmn, x[j]);
+            cmx = q_max(cmx, x[j]);
+          }
+      };
+      if (seg == SEG) body(std::true_type{});
+      else body(std::false_type{});
       __syncthreads();
       if (tid < seg) {
         if (need_norm) {
@@ -445,7 +466,7 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
   }
 }
 
-template <int LH>
+template <int LH, int KINDS>
 __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
                                                              const int32_t* __restrict__ seq_ids,
                                                              const int32_t* __restrict__ cu_new,
@@ -466,7 +487,7 @@ __global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevS
     if (threadIdx.x == 0) set_error(st.err, EPIKV_DEV_CAPACITY);
     return;
   }
-  lag_stream<LH>(st, dm, kv, seq, n_new, layer, kvk, nc0);
+  lag_stream<LH, kLagSeg, false, KINDS>(st, dm, kv, seq, n_new, layer, kvk, nc0);
 }
 
 #ifndef EPIKV_FIN_TILE
@@ -1018,14 +1039,21 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
     const dim3 grid(2 * dm.L, n_seq);
     const int threads = max(32, (dm.H * dm.d / 8 + 31) / 32 * 32);
     auto go = [&](auto kern) { pdl_launch(kern, grid, threads, 0, stream, st, dm, *kv, seq_ids, cu_new, max_new); };
-    switch (dm.d / 8) {
-      case 1: go(lagkv_partial_kernel<1>); break;
-      case 2: go(lagkv_partial_kernel<2>); break;
-      case 4: go(lagkv_partial_kernel<4>); break;
-      case 8: go(lagkv_partial_kernel<8>); break;
-      case 16: go(lagkv_partial_kernel<16>); break;
-      default: go(lagkv_partial_kernel<32>); break;
-    }
+    auto lanes = [&](auto kinds_t) {
+      constexpr int KS = decltype(kinds_t)::value;
+      switch (dm.d / 8) {
+        case 1: go(lagkv_partial_kernel<1, KS>); break;
+        case 2: go(lagkv_partial_kernel<2, KS>); break;
+        case 4: go(lagkv_partial_kernel<4, KS>); break;
+        case 8: go(lagkv_partial_kernel<8, KS>); break;
+        case 16: go(lagkv_partial_kernel<16, KS>); break;
+        default: go(lagkv_partial_kernel<32, KS>); break;
+      }
+    };
+    const int ks = ((dm.kinds & kNormKinds) ? 1 : 0) | ((dm.kinds & kRawKinds) ? 2 : 0);
+    if (ks == 1) lanes(std::integral_constant<int, 1>{});
+    else if (ks == 2) lanes(std::integral_constant<int, 2>{});
+    else lanes(std::integral_constant<int, 0>{});   // both: the runtime flags (fewer spills than both fixed)
     ++*launches;
   }
   {
