@@ -39,7 +39,13 @@
 
 namespace epikv {
 
-constexpr int kSelThreads = 1024;
+#ifndef EPIKV_SEL_THREADS
+// threads of the selection CTA (measured per evicting sequence, 1024 / 512 /
+// 256: one-token decode of 64 sequences 20.7 / 23.9 / 30.7 us; 8,320 slots
+// 26.1 / 29.6 / 43.1 us; 65,536 slots 223 / 300 / 471 us)
+#define EPIKV_SEL_THREADS 1024
+#endif
+constexpr int kSelThreads = EPIKV_SEL_THREADS;
 
 __device__ __forceinline__ uint32_t order_key(float f) {
   if (f != f) return 0u;          // NaN below every number
