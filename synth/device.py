@@ -45,8 +45,9 @@ def load():
 
 
 def upload_2d(dst, dpitch, src, spitch, width, height, ctas, stream=None):
-    """Host-to-device copy of `height` rows of `width` bytes by SM loads of
-    pinned host memory (see synth_upload_2d)."""
+    """Copy of `height` rows of `width` bytes between pinned host memory and
+    device memory (either direction) by SM loads and stores, no copy engine
+    (see synth_upload_2d)."""
     r = load().synth_upload_2d(dst, dpitch, src, spitch, width, height, ctas, _stream(stream))
     if r != 0:
         raise RuntimeError(f"synth_upload_2d failed ({r})")

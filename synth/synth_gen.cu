@@ -189,9 +189,10 @@ __global__ void kv_batch_kernel(uint64_t seed, int n, const int32_t* __restrict_
   *reinterpret_cast<uint4*>(vw.base[kind] + (row + h * d + j0) * 2) = q;
 }
 
-// Delivery of host-resident inputs: row r (of gridDim.y) of `width16` 16-byte
-// vectors, read from pinned host memory through unified addressing by the SMs
-// (no copy engine) and stored to device memory.
+// Delivery of host-resident inputs (and read-back of results): row r (of
+// gridDim.y) of `width16` 16-byte vectors, copied by the SMs through unified
+// addressing (no copy engine), from pinned host memory to device memory or
+// from device memory to pinned host memory.
 __global__ void upload_kernel(char* __restrict__ dst, size_t dpitch, const char* __restrict__ src, size_t spitch,
                               size_t width16) {
   const size_t r = blockIdx.y;
@@ -204,9 +205,10 @@ __global__ void upload_kernel(char* __restrict__ dst, size_t dpitch, const char*
 extern "C" {
 
 // `height` rows of `width` bytes from pinned host memory (rows `spitch` apart)
-// to device memory (rows `dpitch` apart), read by about `ctas` CTAs of SM
-// loads over the host link: the host-to-device input delivery of the
-// end-to-end measurement.  Pointers, pitches and width are 16-byte multiples.
+// to device memory (rows `dpitch` apart), or the other way, copied by about
+// `ctas` CTAs of SM loads and stores over the host link: the input delivery
+// and result read-back of the end-to-end measurement.  Pointers, pitches and
+// width are 16-byte multiples.
 int synth_upload_2d(void* dst, size_t dpitch, const void* src, size_t spitch, size_t width, size_t height, int ctas,
                     cudaStream_t stream) {
   if (!dst || !src || ctas < 1 || (width & 15) || (dpitch & 15) || (spitch & 15) || ((uintptr_t)dst & 15) ||
