@@ -34,11 +34,20 @@
 // layer's kept list in its own slot numbering and a keep bit per union slot
 // (a 32-bit word per 32 slots); layer_union_kernel (a CTA per sequence) turns
 // the keep bits into the new masks and compacts the union's metadata.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
 namespace epikv {
 
+#ifndef EPIKV_SEL_CLUSTER_MIN
+// token budgets: caches of more slots than this take the cluster kernel, the
+// others one CTA per sequence (measured per evicting sequence, one CTA /
+// cluster of 8: 8,320 slots 26 / 54 us, a one-token ragged eviction 21 /
+// 39 us, 2,048 slots 14 / 32 us; 4 x 65,536 slots 218 / 70 us)
+#define EPIKV_SEL_CLUSTER_MIN 24576
+#endif
 #ifndef EPIKV_SEL_THREADS
 // threads of the selection CTA (measured per evicting sequence, 1024 / 512 /
 // 256: one-token decode of 64 sequences 20.7 / 23.9 / 30.7 us; 8,320 slots
@@ -377,6 +386,239 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   }
 }
 
+// ---------------------------------------------------------------- token budgets on a thread-block cluster
+//
+// One sequence's selection spread over a cluster of kCluCtas CTAs (DSMEM for
+// the merges, cluster barriers between phases; every CTA of a cluster takes
+// the same path, so none leaves while the others wait).  The sequence's slots
+// [0, n) are cut into one contiguous slice per CTA.  The radix passes count
+// each slice's candidate keys into the CTA's own 256-bin histogram (double
+// buffered: a pass's bins are read by the other CTAs until the next pass's
+// barrier); after the barrier every CTA reads all kCluCtas histograms and
+// takes the same decision.  The ordered scans publish each CTA's counts (keys
+// equal to the threshold, kept slots, first evicted slot) for the others'
+// prefixes.  The slot metadata is compacted in rounds of destination rows:
+// every CTA stages its part of the round's sources, a barrier, then the
+// writes (a round's sources lie at or after its destinations' end, so they
+// are not written by the round).  Results equal select_kernel's bit for bit.
+constexpr int kCluCtas = 8;
+constexpr int kCluThreads = 512;
+constexpr int kCluStageWords = 8192;   // 32 KiB: a slice's staged keys, then a round's metadata
+
+struct CluShared {
+  uint32_t hist[2][256];
+  uint32_t prefix, mask, remaining;
+  int pub[3];        // this CTA's equal-key count, kept count, first evicted slot
+  int sh_scan[32];
+};
+
+__global__ void __cluster_dims__(kCluCtas, 1, 1) __launch_bounds__(kCluThreads)
+    select_cluster_kernel(DevState st, Dims dm, const int32_t* __restrict__ seq_ids,
+                          const int32_t* __restrict__ budget, const int32_t* __restrict__ trigger,
+                          int32_t* __restrict__ kept_out, int kept_stride, int32_t* __restrict__ n_kept_out) {
+  pdl_wait();
+  pdl_trigger();
+  namespace cg = cooperative_groups;
+  cg::cluster_group cluster = cg::this_cluster();
+  constexpr int NT = kCluThreads;
+  const int rank = (int)cluster.block_rank();
+  const int b = blockIdx.x / kCluCtas, tid = threadIdx.x;
+  const bool lead = rank == 0 && tid == 0;
+  const int seq = seq_ids[b];
+  if (seq < 0 || seq >= dm.S) {
+    if (lead) set_error(st.err, EPIKV_DEV_BATCH);
+    return;
+  }
+  const int n = st.n_cache[seq];
+  const int K = budget[b];
+  if (K < 1 || K > dm.T) {
+    if (lead) {
+      set_error(st.err, EPIKV_DEV_BUDGET);
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const int trig = trigger ? trigger[b] : K;
+  if (n <= K || n <= trig) {  // nothing to evict
+    if (lead) {
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const int P = min(st.prefill[seq], n);
+  const int R = min(min(dm.recency_cap, K / 4), max(0, K - P));
+  const int M = max(0, K - P - R);
+  const int c0 = P, c1 = n - R;  // candidates [c0, c1)
+  if (max(K, P) > kept_stride) {
+    if (lead) {
+      set_error(st.err, EPIKV_DEV_KEPT);
+      st.first_changed[seq] = n;
+      if (n_kept_out) n_kept_out[b] = n;
+    }
+    return;
+  }
+  const float* __restrict__ sc = st.score[kind_index(st.policy[seq])] + (size_t)seq * dm.T;
+  int32_t* out = kept_out + (size_t)b * kept_stride;
+  __shared__ CluShared cs;
+  extern __shared__ uint32_t stage[];   // kCluStageWords
+
+  // this CTA's slice of the slots and its candidates
+  const int s0 = (int)((int64_t)n * rank / kCluCtas), s1 = (int)((int64_t)n * (rank + 1) / kCluCtas);
+  const int a0 = max(s0, c0), a1 = max(a0, min(s1, c1));
+  const bool staged = a1 - a0 <= kCluStageWords;
+  if (staged) {
+    for (int i = a0 + tid; i < a1; i += NT) stage[i - a0] = order_key(sc[i]);
+    __syncthreads();
+  }
+  auto key_at = [&](int i) -> uint32_t { return staged ? stage[i - a0] : order_key(sc[i]); };
+
+  // ---- radix select of the M-th largest candidate key over the cluster
+  uint32_t prefix = 0u, mask = 0u, remaining = (uint32_t)M;
+  if (M > 0) {
+    for (int pass = 0, shift = 24; shift >= 0; ++pass, shift -= 8) {
+      uint32_t* h = cs.hist[pass & 1];
+      for (int j = tid; j < 256; j += NT) h[j] = 0u;
+      __syncthreads();
+      for (int i = a0 + tid; i < a1; i += NT) {
+        const uint32_t k = key_at(i);
+        if ((k & mask) == prefix) atomicAdd(&h[(k >> shift) & 255u], 1u);
+      }
+      cluster.sync();   // every CTA's bins of this pass are complete
+      if (tid < 32) {
+        // lane l owns digits 255-8l .. 248-8l (descending), summed over the cluster
+        const int lane = tid;
+        uint32_t cnt[8], lsum = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cnt[j] = 0;
+        for (int r = 0; r < kCluCtas; ++r) {
+          const uint32_t* hr = cluster.map_shared_rank(h, r);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) cnt[j] += hr[255 - 8 * lane - j];
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) lsum += cnt[j];
+        uint32_t incl = lsum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const unsigned hit = __ballot_sync(0xffffffffu, incl >= remaining);
+        const int owner = __ffs(hit) - 1;  // first lane reaching the target
+        if (lane == owner) {
+          uint32_t before = incl - lsum;
+          for (int j = 0; j < 8; ++j) {
+            if (before + cnt[j] >= remaining) {
+              cs.prefix = prefix | ((uint32_t)(255 - 8 * lane - j) << shift);
+              cs.mask = mask | (255u << shift);
+              cs.remaining = remaining - before;
+              break;
+            }
+            before += cnt[j];
+          }
+        }
+      }
+      __syncthreads();
+      prefix = cs.prefix;
+      mask = cs.mask;
+      remaining = cs.remaining;
+    }
+  }
+  const uint32_t theta = M > 0 ? prefix : 0xFFFFFFFFu;
+  const int need_eq = M > 0 ? (int)remaining : 0;
+
+  // ---- ordered scans: contiguous per-thread ranges of the slice, CTA
+  // prefixes from the lower ranks' published counts
+  const int per = (s1 - s0 + NT - 1) / NT;
+  const int ta = min(s1, s0 + tid * per), te = min(s1, ta + per);
+  int eq_local = 0;
+  for (int i = max(ta, c0); i < min(te, c1); ++i) eq_local += (key_at(i) == theta);
+  int eq_cta;
+  int eqs = block_exclusive_scan<NT>(eq_local, &eq_cta, cs.sh_scan);
+  if (tid == 0) cs.pub[0] = eq_cta;
+  cluster.sync();
+  for (int r = 0; r < rank; ++r) eqs += cluster.map_shared_rank(cs.pub, r)[0];
+  int keep_local = 0, first_ev = INT_MAX;
+  {
+    int e = eqs;
+    for (int i = ta; i < te; ++i) {
+      bool keep = (i < c0) || (i >= c1);
+      if (!keep) {
+        const uint32_t k = key_at(i);
+        keep = k > theta || (k == theta && e++ < need_eq);
+      }
+      if (keep) ++keep_local; else first_ev = min(first_ev, i);
+    }
+  }
+  int keep_cta;
+  int o = block_exclusive_scan<NT>(keep_local, &keep_cta, cs.sh_scan);
+  const int fe_cta = block_min<NT>(first_ev, cs.sh_scan);
+  if (tid == 0) {
+    cs.pub[1] = keep_cta;
+    cs.pub[2] = fe_cta;
+  }
+  cluster.sync();
+  int n_kept = 0, fe = INT_MAX;
+  for (int r = 0; r < kCluCtas; ++r) {
+    const int* pr = cluster.map_shared_rank(cs.pub, r);
+    if (r < rank) o += pr[1];
+    n_kept += pr[1];
+    fe = min(fe, pr[2]);
+  }
+  fe = min(fe, n_kept);
+  {
+    int e = eqs;
+    for (int i = ta; i < te; ++i) {
+      bool keep = (i < c0) || (i >= c1);
+      if (!keep) {
+        const uint32_t k = key_at(i);
+        keep = k > theta || (k == theta && e++ < need_eq);
+      }
+      if (keep) out[o++] = i;
+    }
+  }
+  cluster.sync();   // the whole kept list is written and visible to the cluster (and no DSMEM read is pending)
+
+  // ---- slot metadata in place, in rounds of destination rows
+  int32_t* ps = st.pos + (size_t)seq * dm.T;
+  const size_t base = (size_t)seq * dm.T;
+  unsigned on = 0;
+#pragma unroll
+  for (int k = 0; k < kNumKinds; ++k) on |= (st.score[k] != nullptr ? 1u : 0u) << k;
+  const int n_on = __popc(on);
+  const int rpc = kCluStageWords / (n_on + 1);   // rows of a CTA per round
+  for (int j0 = fe; j0 < n_kept; j0 += kCluCtas * rpc) {
+    const int r0 = j0 + rank * rpc, r1 = min(n_kept, r0 + rpc);
+    for (int j = r0 + tid; j < r1; j += NT) {
+      const int src = out[j];
+      int q = 0;
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k)
+        if (on >> k & 1u) stage[(q++) * rpc + (j - r0)] = __float_as_uint(st.score[k][base + src]);
+      stage[n_on * rpc + (j - r0)] = (uint32_t)ps[src];
+    }
+    cluster.sync();   // every source of the round is read before any of its rows is written
+    for (int j = r0 + tid; j < r1; j += NT) {
+      int q = 0;
+#pragma unroll
+      for (int k = 0; k < kNumKinds; ++k)
+        if (on >> k & 1u) st.score[k][base + j] = __uint_as_float(stage[(q++) * rpc + (j - r0)]);
+      ps[j] = (int32_t)stage[n_on * rpc + (j - r0)];
+    }
+    __syncthreads();  // the stage is reused by the next round
+  }
+  if (lead) {
+    st.n_cache[seq] = n_kept;
+    st.first_changed[seq] = fe;
+    if (n_kept_out) n_kept_out[b] = n_kept;
+    atomicAdd(&st.stats[1], 1ull);
+    atomicAdd(&st.stats[2], (unsigned long long)(n_kept - fe));
+    atomicAdd(&st.stats[3], (unsigned long long)(n_kept - fe) * (unsigned long long)dm.L);
+  }
+}
+
 constexpr int kLayerThreads = 256;
 
 // What both per-layer kernels derive from a sequence's layer budgets.
@@ -679,6 +921,9 @@ cudaError_t launch_select(const DevState& st, const Dims& dm, int n_seq, const i
   } else if (dm.select_chunk > 1) {
     pdl_launch(select_kernel<true>, n_seq, kSelThreads, smem, stream, st, dm, seq_ids, budget, trigger, kept,
                kept_stride, n_kept, sel_staged_cap(dm), words);
+  } else if (dm.T > EPIKV_SEL_CLUSTER_MIN) {
+    pdl_launch(select_cluster_kernel, n_seq * kCluCtas, kCluThreads, (size_t)kCluStageWords * sizeof(uint32_t),
+               stream, st, dm, seq_ids, budget, trigger, kept, kept_stride, n_kept);
   } else {
     pdl_launch(select_kernel<false>, n_seq, kSelThreads, smem, stream, st, dm, seq_ids, budget, trigger, kept,
                kept_stride, n_kept, sel_staged_cap(dm), words);

@@ -221,7 +221,7 @@ def kernel_short_name(name):
     mangled) kernel name: the function's identifier only."""
     import re
     for ident in ("bandz_g_kernel", "bandz_token_kernel", "lagkv_partial_kernel", "score_finalize_kernel",
-                  "token_kernel", "select_kernel", "layer_keep_kernel", "layer_union_kernel", "compact_stash_kernel",
+                  "token_kernel", "select_cluster_kernel", "select_kernel", "layer_keep_kernel", "layer_union_kernel", "compact_stash_kernel",
                   "compact_consumed_kernel", "compact_kernel"):
         if re.search(r"(?<![A-Za-z_])" + ident, name):
             return ident

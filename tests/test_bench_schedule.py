@@ -61,3 +61,15 @@ def test_stream_bytes_and_kernel_table():
     assert t["compact_kernel"]["launches_per_step"] == 1 and t["compact_kernel"]["ms_per_step"] == 3.0
     assert t["compact_kernel"]["gbs"] == pytest.approx(1000.0) and t["compact_kernel"]["hbm_frac"] == pytest.approx(1 / 6)
     assert "gbs" not in t["select_kernel"]
+
+
+def test_kernel_short_names():
+    from paper_2606_26472_gb300 import epikv as E
+    assert E.kernel_short_name("_ZN5epikv12token_kernelILi16EEEvNS_8DevStateE") == "token_kernel"
+    assert E.kernel_short_name("_ZN5epikv18bandz_token_kernelILi2EEEv") == "bandz_token_kernel"
+    assert E.kernel_short_name("void epikv::compact_kernel<false, true>(epikv::DevState)") == "compact_kernel"
+    assert E.kernel_short_name("_ZN5epikv20compact_stash_kernelEv") == "compact_stash_kernel"
+    assert E.kernel_short_name("_ZN5epikv23compact_consumed_kernelE") == "compact_consumed_kernel"
+    assert E.kernel_short_name("_ZN5epikv21select_cluster_kernelENS_8DevStateE") == "select_cluster_kernel"
+    assert E.kernel_short_name("_ZN5epikv13select_kernelILb0EEEv") == "select_kernel"
+    assert E.kernel_short_name("something_else") == "something_else"
