@@ -580,6 +580,10 @@ def run_ours(args):
                 upload_2d(pool[0, lo_i].data_ptr(), pitch, src[kind].data_ptr(), plane, plane, L, up_ctas, copy_stream)
             copied[i].record(copy_stream)
 
+        # the copy kernel's first launch (module load, first transfers) before timing
+        for kind, pool in ((0, cache.k), (1, cache.v)):
+            upload_2d(pool[0, e2e_base + Bn * fresh].data_ptr(), pitch, payload[0][kind].data_ptr(), plane, plane, L,
+                      up_ctas, copy_stream)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
