@@ -370,15 +370,26 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
       // per-token conditions compile away; the arithmetic is the same
       auto body = [&](auto full_t) {
         constexpr bool FULL = decltype(full_t)::value;
-        bool bad = false;
+        int64_t offs[SEG];
+        bool all_ok = active;
 #pragma unroll
         for (int j = 0; j < SEG; ++j) {
-          const bool take = (FULL || j < seg) && active;
-          const int64_t off = take ? soff[i + j] : 0;
-          bad |= off < 0;
-          x[j] = ld_stream16_if(kvb_ch + off * 2, take && off >= 0);
+          offs[j] = (FULL || j < seg) ? soff[i + j] : 0;
+          all_ok &= offs[j] >= 0;
         }
-        if (bad) set_error(st.err, EPIKV_DEV_SLOT);
+        if (FULL && all_ok) {  // every row of the segment mapped: plain loads
+#pragma unroll
+          for (int j = 0; j < SEG; ++j) x[j] = ld_stream16(kvb_ch + offs[j] * 2);
+        } else {
+          bool bad = false;
+#pragma unroll
+          for (int j = 0; j < SEG; ++j) {
+            const bool take = (FULL || j < seg) && active;
+            bad |= take && offs[j] < 0;
+            x[j] = ld_stream16_if(kvb_ch + offs[j] * 2, take && offs[j] >= 0);
+          }
+          if (bad) set_error(st.err, EPIKV_DEV_SLOT);
+        }
         if (need_raw) {  // population variance of the stored vector over the head dimension
 #pragma unroll
           for (int j = 0; j < SEG; ++j) {
