@@ -177,10 +177,20 @@ __global__ void __launch_bounds__(kGThreads, (EPIKV_G_MINB > 0 ? EPIKV_G_MINB : 
 #define EPIKV_LAG_SEG 8
 #endif
 #ifndef EPIKV_LAG_MINB
-#define EPIKV_LAG_MINB 3  // caps registers at 80 (measured best with 8-token segments)
+#define EPIKV_LAG_MINB 3  // with EPIKV_LAG_MAXREG 0: registers capped at 80
+#endif
+#ifndef EPIKV_LAG_PF
+#define EPIKV_LAG_PF 1  // measured: 1 segment ahead 110 us, none 115 us, 2 ahead 119 us
 #endif
 constexpr int kLagSeg = EPIKV_LAG_SEG;  // tokens per segment (never crosses a chunk boundary)
+constexpr int kLagPf = EPIKV_LAG_PF;    // a row is prefetched into L2 this many segments ahead
 constexpr int kLagOffs = 256;   // slot offsets looked up per group of tokens
+
+// Fire-and-forget bulk prefetch of [p, p + bytes) into L2 (p 16-byte aligned,
+// bytes a multiple of 16).
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(p), "r"(bytes) : "memory");
+}
 
 __device__ __forceinline__ uint32_t bf16x2_min(uint32_t a, uint32_t b) {
   __nv_bfloat162 r = __hmin2(*reinterpret_cast<__nv_bfloat162*>(&a), *reinterpret_cast<__nv_bfloat162*>(&b));
@@ -213,6 +223,7 @@ __device__ __forceinline__ float f2_lo(f32x2 v) {
 __device__ __forceinline__ float f2_hi(f32x2 v) {
   float lo, hi;
   asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  (void)lo;
   return hi;
 }
 __device__ __forceinline__ f32x2 f2_fma(f32x2 a, f32x2 b, f32x2 c) {
@@ -332,15 +343,20 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
   const bool need_raw = KINDS ? (KINDS & 2) != 0 : (dm.kinds & kRawKinds) != 0;
   __nv_bfloat16* rng = need_norm ? st.lag_rng + ((((size_t)seq * dm.L + layer) * 2 + kvk) * 4) * hd : nullptr;
 
-  uint4 pmn = make_uint4(0, 0, 0, 0), pmx = pmn, cmn = pmn, cmx = pmn;
-  if (active && need_norm) {
-    pmn = *reinterpret_cast<const uint4*>(rng + 0 * hd + ch);
-    pmx = *reinterpret_cast<const uint4*>(rng + 1 * hd + ch);
-    cmn = *reinterpret_cast<const uint4*>(rng + 2 * hd + ch);
-    cmx = *reinterpret_cast<const uint4*>(rng + 3 * hd + ch);
-  }
+  // the previous chunk's range lives on only as its affine map; it is written
+  // back as soon as a chunk completes, the running range at the end
+  uint4 cmn = make_uint4(0, 0, 0, 0), cmx = cmn;
   f32x2 na[4], nc[4];
-  prev_affine(pmn, pmx, dm.lag_eps, na, nc);
+  {
+    uint4 pmn = cmn, pmx = cmn;
+    if (active && need_norm) {
+      pmn = *reinterpret_cast<const uint4*>(rng + 0 * hd + ch);
+      pmx = *reinterpret_cast<const uint4*>(rng + 1 * hd + ch);
+      cmn = *reinterpret_cast<const uint4*>(rng + 2 * hd + ch);
+      cmx = *reinterpret_cast<const uint4*>(rng + 3 * hd + ch);
+    }
+    prev_affine(pmn, pmx, dm.lag_eps, na, nc);
+  }
 
   const float inv_d = 1.f / (float)dm.d;
   const char* kvbase = kvk ? kv.base[1] : kv.base[0];  // a select: no local copy of the parameter struct
@@ -362,6 +378,13 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
     __syncthreads();
     for (int t = tid; t < gn; t += nthr) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
     __syncthreads();
+    // rows are prefetched into L2 kLagPf segments ahead of their loads (whole
+    // rows of H*d channels, one bulk prefetch each); the group's first ones here
+    const uint32_t row_bytes = (uint32_t)hd * 2u;
+    if constexpr (SEG > 1 && kLagPf > 0) {
+      for (int t = tid; t < min(kLagPf * SEG, gn); t += nthr)
+        if (soff[t] >= 0) prefetch_l2_bulk(kvbase + soff[t] * 2, row_bytes);
+    }
     for (int i = 0; i < gn;) {
       const int seg = min(min(dm.lag - r, gn - i), SEG);
       const bool has_prev = p0 + g0 + i >= dm.lag;   // the segment's chunk is not chunk 0
@@ -390,10 +413,23 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
           }
           if (bad) set_error(st.err, EPIKV_DEV_SLOT);
         }
-        if (need_raw) {  // population variance of the stored vector over the head dimension
+        if constexpr (SEG > 1 && kLagPf > 0) {  // rows [i + kLagPf*SEG, + seg): every row once over the group
+          const int t = i + kLagPf * SEG + tid;
+          if (tid < seg && t < gn && soff[t] >= 0) prefetch_l2_bulk(kvbase + soff[t] * 2, row_bytes);
+        }
+        // token by token, so that a row's registers are free once it is used:
+        // its raw variance, its normalised moments and the running range
+        const bool moments = has_prev && need_norm;  // uniform across the block
+        float v[NV];
+        if (r == 0) {
+          cmn = x[0];
+          cmx = x[0];
+        }
 #pragma unroll
-          for (int j = 0; j < SEG; ++j) {
-            if (FULL || j < seg) {
+        for (int j = 0; j < SEG; ++j) {
+          v[2 * j] = v[2 * j + 1] = 0.f;
+          if (FULL || j < seg) {
+            if (need_raw) {  // population variance of the stored vector over the head dimension
               float xf[8], s1 = 0.f;
               unpack8(x[j], xf);
 #pragma unroll
@@ -408,15 +444,12 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
               const float var_raw = group_sum(s2, LH) * inv_d;
               if (q == 0 && active) hr[parity][j][h] = var_raw;
             }
+            if (moments) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
+            cmn = q_min(cmn, x[j]);
+            cmx = q_max(cmx, x[j]);
           }
         }
-        if (has_prev && need_norm) {  // uniform across the block
-          float v[NV];
-#pragma unroll
-          for (int j = 0; j < SEG; ++j) {
-            v[2 * j] = v[2 * j + 1] = 0.f;
-            if (FULL || j < seg) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
-          }
+        if (moments) {
           transpose_sum<LH / 2, NV, NV>(v, tid & 31);
           if (active) {
             if constexpr (LH <= NV) {
@@ -427,17 +460,6 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
             }
           }
         }
-        // advance the running range of the current chunk
-        if (r == 0) {
-          cmn = x[0];
-          cmx = x[0];
-        }
-#pragma unroll
-        for (int j = 0; j < SEG; ++j)
-          if (FULL || j < seg) {
-            cmn = q_min(cmn, x[j]);
-            cmx = q_max(cmx, x[j]);
-          }
       };
       if (seg == SEG) body(std::true_type{});
       else body(std::false_type{});
@@ -461,24 +483,32 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
       parity ^= 1;
       r += seg;
       if (r == dm.lag) {  // chunk complete: it becomes the previous chunk
-        pmn = cmn;
-        pmx = cmx;
-        prev_affine(pmn, pmx, dm.lag_eps, na, nc);
+        prev_affine(cmn, cmx, dm.lag_eps, na, nc);
+        if (active && need_norm) {
+          *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = cmn;
+          *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = cmx;
+        }
         r = 0;
       }
       i += seg;
     }
   }
   if (active && need_norm) {
-    *reinterpret_cast<uint4*>(rng + 0 * hd + ch) = pmn;
-    *reinterpret_cast<uint4*>(rng + 1 * hd + ch) = pmx;
     *reinterpret_cast<uint4*>(rng + 2 * hd + ch) = cmn;
     *reinterpret_cast<uint4*>(rng + 3 * hd + ch) = cmx;
   }
 }
 
+#ifndef EPIKV_LAG_MAXREG
+#define EPIKV_LAG_MAXREG 72  // 7 CTAs of 128 threads per SM: 2,048 CTAs in two rounds (measured best; 64 spills)
+#endif
+#if EPIKV_LAG_MAXREG > 0
+#define EPIKV_LAG_BOUNDS __maxnreg__(EPIKV_LAG_MAXREG)
+#else
+#define EPIKV_LAG_BOUNDS __launch_bounds__(256, EPIKV_LAG_MINB)
+#endif
 template <int LH, int KINDS>
-__global__ void __launch_bounds__(256, EPIKV_LAG_MINB) lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
+__global__ void EPIKV_LAG_BOUNDS lagkv_partial_kernel(DevState st, Dims dm, KvDev kv,
                                                              const int32_t* __restrict__ seq_ids,
                                                              const int32_t* __restrict__ cu_new,
                                                              int max_new) {
