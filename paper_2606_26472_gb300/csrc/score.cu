@@ -215,17 +215,8 @@ __device__ __forceinline__ f32x2 f2_pack(float lo, float hi) {
   asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
   return d;
 }
-__device__ __forceinline__ float f2_lo(f32x2 v) {
-  float lo, hi;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-  return lo;
-}
-__device__ __forceinline__ float f2_hi(f32x2 v) {
-  float lo, hi;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-  (void)lo;
-  return hi;
-}
+__device__ __forceinline__ float f2_lo(f32x2 v) { return __uint_as_float((unsigned)(v & 0xffffffffull)); }
+__device__ __forceinline__ float f2_hi(f32x2 v) { return __uint_as_float((unsigned)(v >> 32)); }
 __device__ __forceinline__ f32x2 f2_fma(f32x2 a, f32x2 b, f32x2 c) {
   f32x2 d;
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
@@ -391,8 +382,9 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
       uint4 x[SEG];
       // FULL: every token of the segment is taken (the common case), so the
       // per-token conditions compile away; the arithmetic is the same
-      auto body = [&](auto full_t) {
+      auto body = [&](auto full_t, auto mom_t) {
         constexpr bool FULL = decltype(full_t)::value;
+        constexpr bool MOM = decltype(mom_t)::value;  // has_prev && need_norm: the normalised moments
         int64_t offs[SEG];
         bool all_ok = active;
 #pragma unroll
@@ -417,39 +409,48 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
           const int t = i + kLagPf * SEG + tid;
           if (tid < seg && t < gn && soff[t] >= 0) prefetch_l2_bulk(kvbase + soff[t] * 2, row_bytes);
         }
-        // token by token, so that a row's registers are free once it is used:
-        // its raw variance, its normalised moments and the running range
-        const bool moments = has_prev && need_norm;  // uniform across the block
+        // two tokens at a time, so that rows' registers are free once used:
+        // their raw variances, their normalised moments, then the running
+        // range over both (the same min/max sequence as token by token)
         float v[NV];
         if (r == 0) {
           cmn = x[0];
           cmx = x[0];
         }
 #pragma unroll
-        for (int j = 0; j < SEG; ++j) {
-          v[2 * j] = v[2 * j + 1] = 0.f;
-          if (FULL || j < seg) {
-            if (need_raw) {  // population variance of the stored vector over the head dimension
-              float xf[8], s1 = 0.f;
-              unpack8(x[j], xf);
+        for (int j0 = 0; j0 < SEG; j0 += 2) {
 #pragma unroll
-              for (int e = 0; e < 8; ++e) s1 += xf[e];
-              const float mean = group_sum(s1, LH) * inv_d;
-              float s2 = 0.f;
+          for (int j = j0; j < j0 + 2 && j < SEG; ++j) {
+            if (FULL || j < seg) {
+              if (need_raw) {  // population variance of the stored vector over the head dimension
+                float xf[8], s1 = 0.f;
+                unpack8(x[j], xf);
 #pragma unroll
-              for (int e = 0; e < 8; ++e) {
-                const float dv = xf[e] - mean;
-                s2 = fmaf(dv, dv, s2);
+                for (int e = 0; e < 8; ++e) s1 += xf[e];
+                const float mean = group_sum(s1, LH) * inv_d;
+                float s2 = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  const float dv = xf[e] - mean;
+                  s2 = fmaf(dv, dv, s2);
+                }
+                const float var_raw = group_sum(s2, LH) * inv_d;
+                if (q == 0 && active) hr[parity][j][h] = var_raw;
               }
-              const float var_raw = group_sum(s2, LH) * inv_d;
-              if (q == 0 && active) hr[parity][j][h] = var_raw;
+              if constexpr (MOM) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
+            } else if constexpr (MOM) {
+              v[2 * j] = v[2 * j + 1] = 0.f;
             }
-            if (moments) lag_moments(x[j], na, nc, v[2 * j], v[2 * j + 1]);
-            cmn = q_min(cmn, x[j]);
-            cmx = q_max(cmx, x[j]);
+          }
+          if (j0 + 1 < SEG && (FULL || j0 + 1 < seg)) {
+            cmn = q_min(q_min(cmn, x[j0]), x[j0 + 1]);
+            cmx = q_max(q_max(cmx, x[j0]), x[j0 + 1]);
+          } else if (FULL || j0 < seg) {
+            cmn = q_min(cmn, x[j0]);
+            cmx = q_max(cmx, x[j0]);
           }
         }
-        if (moments) {
+        if constexpr (MOM) {
           transpose_sum<LH / 2, NV, NV>(v, tid & 31);
           if (active) {
             if constexpr (LH <= NV) {
@@ -461,8 +462,13 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
           }
         }
       };
-      if (seg == SEG) body(std::true_type{});
-      else body(std::false_type{});
+      if (has_prev && need_norm) {
+        if (seg == SEG) body(std::true_type{}, std::true_type{});
+        else body(std::false_type{}, std::true_type{});
+      } else {
+        if (seg == SEG) body(std::true_type{}, std::false_type{});
+        else body(std::false_type{}, std::false_type{});
+      }
       __syncthreads();
       if (tid < seg) {
         if (need_norm) {
