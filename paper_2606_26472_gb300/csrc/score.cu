@@ -829,7 +829,7 @@ __device__ __forceinline__ void band_token_scores(const DevState& st, const Dims
 // one thread (the warp first loads them into shared memory together, so the
 // sum waits on one round of loads, not on 2L); its rolling mean over this u
 // and the ring's earlier ones, a lane per window position in the same order,
-// the same warp sum.  Warp 0 calls it.
+// the same warp sum.  One warp calls it.
 __device__ __forceinline__ void kv_token_scores(const DevState& st, const Dims& dm, int seq, int nc0, int pos) {
   const int lane = threadIdx.x & 31;
   __shared__ float pv[2 * 64];  // the host admits at most 64 layers
@@ -928,8 +928,8 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
   if (!s_last) return;
   __threadfence();
   extern __shared__ float win[];  // [nb][z_window]
-  band_token_scores(st, dm, seq, nc0, pos, win);
-  if (tid == 0) token_commit(st, dm, seq, nc0, pos);
+  band_token_scores(st, dm, seq, nc0, pos, win);  // warp 0 after a block barrier
+  if (tid == 32) token_commit(st, dm, seq, nc0, pos);  // meanwhile: they touch disjoint state
 }
 
 // One new token per sequence with a K/V kind (and any band kinds): the whole
@@ -985,9 +985,11 @@ __global__ void __launch_bounds__(kGThreads, EPIKV_TOKEN_MINB) token_kernel(DevS
   if (!s_last) return;
   __threadfence();
   extern __shared__ float win[];  // [nb][z_window] (band kinds)
+  // three warps at once, on disjoint state: the band scores (warp 0, after a
+  // block barrier), the K/V scores (warp 1) and the commit (warp 2)
   if (nbc) band_token_scores(st, dm, seq, nc0, pos, win);
-  if (tid < 32) kv_token_scores(st, dm, seq, nc0, pos);
-  if (tid == 0) token_commit(st, dm, seq, nc0, pos);
+  if (tid >= 32 && tid < 64) kv_token_scores(st, dm, seq, nc0, pos);
+  if (tid == 64) token_commit(st, dm, seq, nc0, pos);
 }
 
 // ------------------------------------------------------------------ launchers
