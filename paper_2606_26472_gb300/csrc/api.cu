@@ -120,6 +120,7 @@ size_t carve(const Dims& d, DevState* st, char* base) {
     const size_t nb = d.nA + d.nB;
     st->h_prev = (__nv_bfloat16*)take(S * 2 * nb * d.D * 2);
     st->g_ring = (float*)take(S * nb * d.G * 4);
+    st->ztok = (float*)take(S * 2 * nb * 4);
   }
   if (d.kinds & kNormKinds) {
     st->lag_rng = (__nv_bfloat16*)take(S * d.L * 2 * 4 * (size_t)d.H * d.d * 2);

@@ -47,6 +47,7 @@ struct DevState {
   int32_t* pos;            // [S][T] position of each slot
   __nv_bfloat16* h_prev;   // [S][2][n_band][D] last hidden row per band layer
   float* g_ring;           // [S][n_band][G] g by position (mod G)
+  float* ztok;             // [S][2][n_band] a decode step's per-band z and window mean of g (band kinds)
   __nv_bfloat16* lag_rng;  // [S][L][2][4][H][d] prev min, prev max, cur min, cur max
   float* lag_part;         // [S][max_new][2L] per-(layer, K|V) head-summed normalised variances
   float* raw_part;         // [S][max_new][2L] per-(layer, K|V) head-summed raw variances

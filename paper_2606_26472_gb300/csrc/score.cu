@@ -707,21 +707,27 @@ __global__ void __launch_bounds__(kFinThreads) score_finalize_kernel(DevState st
   }
 }
 
-
 // ---- one new token per sequence (a decode step)
 #ifndef EPIKV_TOKEN_MINB
 // token_kernel CTAs resident per SM: 5 caps registers at 48 (64 ragged
 // sequences' decode step: 45.7 / 41.1 / 38.5 / 38.5 us at 3 / 4 / 5 / 6)
 #define EPIKV_TOKEN_MINB 5
 #endif
-//
-// The band g of one (band layer, sequence): the new row against the previous
-// one (h_prev), exactly as bandz_g_kernel forms it (same per-thread vectors,
-// warp sums and fixed-order cross-warp sum); writes the ring and h_prev.
-// Every thread of a kGThreads block calls it.
+
+// One new token's g for one band layer (Eq. 1), from its row and the saved
+// previous row (h_prev), exactly as bandz_g_kernel forms it (same per-thread
+// vectors, fused multiply-adds, warp sums and fixed-order cross-warp sum);
+// the row is saved as the next call's previous row.  Then, for the band
+// kinds' scores (Eq. 3), this band's z of the new g against its window and
+// the window's mean, with score_finalize_kernel's arithmetic and order (the
+// shifted two-pass over g at positions pos, pos-1, ..., pos-n+1, one thread),
+// stored per (sequence, band) for the last CTA to combine.  The window's
+// earlier values are loaded with the rows into `win` (z_window floats of
+// shared memory).  Every thread of a kGThreads block calls it.
 template <int VPT>
 __device__ __forceinline__ void band_token_g(const DevState& st, const Dims& dm, const BandRows& rows,
-                                             int64_t row_stride, int band, int seq, int r0, int pos, int par) {
+                                             int64_t row_stride, int band, int seq, int r0, int pos, int par,
+                                             float* win) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nb = dm.nA + dm.nB;
   const int VR = dm.D >> 3;
@@ -729,6 +735,8 @@ __device__ __forceinline__ void band_token_g(const DevState& st, const Dims& dm,
   const __nv_bfloat16* cur = rows.p[band] + (int64_t)r0 * row_stride;
   const __nv_bfloat16* prow = st.h_prev + ((size_t)(seq * 2 + par) * nb + band) * dm.D;
   __nv_bfloat16* hp_wr = st.h_prev + ((size_t)(seq * 2 + (par ^ 1)) * nb + band) * dm.D;
+  float* ring = st.g_ring + ((size_t)seq * nb + band) * dm.G;
+  const int n = pos >= 1 ? min(dm.z_window, pos) : 0;  // the new g's window, itself included
   uint4 c[VPT], p[VPT];
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
@@ -736,6 +744,7 @@ __device__ __forceinline__ void band_token_g(const DevState& st, const Dims& dm,
     c[k] = v < VR ? ld_stream16(cur + v * 8) : make_uint4(0, 0, 0, 0);
     p[k] = v < VR ? ld_stream16(prow + v * 8) : make_uint4(0, 0, 0, 0);
   }
+  for (int k = 1 + tid; k < n; k += kGThreads) win[k] = __ldcg(ring + ((pos - k) & (dm.G - 1)));
   float acc = 0.f;
 #pragma unroll
   for (int k = 0; k < VPT; ++k) {
@@ -760,53 +769,54 @@ __device__ __forceinline__ void band_token_g(const DevState& st, const Dims& dm,
     float sum = 0.f;
 #pragma unroll
     for (int w = 0; w < kGThreads / 32; ++w) sum += red[w];
-    if (pos >= 1) st.g_ring[((size_t)seq * (dm.nA + dm.nB) + band) * dm.G + (pos & (dm.G - 1))] = sqrtf(sum);
+    const float g = sqrtf(sum);
+    if (pos >= 1) ring[pos & (dm.G - 1)] = g;
+    if (n > 0) {
+      win[0] = g;
+      const float* row = win;  // row[k] = g at position pos - k
+      float z = 0.f, gbar = 0.f;
+      if (dm.kinds & EPIKV_SCORE_BANDZ) {
+        const float gnew = row[0];
+        float dsum = 0.f;
+        for (int k = 0; k < n; ++k) dsum += row[k] - gnew;
+        const float mean_d = dsum / (float)n;
+        float dev = 0.f;
+        for (int k = 0; k < n; ++k) {
+          const float e = (row[k] - gnew) - mean_d;
+          dev = fmaf(e, e, dev);
+        }
+        const float sigma = sqrtf(dev / (float)n);
+        z = -mean_d / (sigma + dm.z_eps);
+      }
+      if (dm.kinds & EPIKV_SCORE_HSVAR) {
+        float s = 0.f;
+        for (int k = 0; k < n; ++k) s += row[k];
+        gbar = s / (float)n;
+      }
+      st.ztok[(size_t)(seq * 2) * nb + band] = z;
+      st.ztok[(size_t)(seq * 2 + 1) * nb + band] = gbar;
+    }
   }
 }
 
-// The band kinds' scores of the new token at slot nc0: every band's window
-// staged from the ring in `win` ([nb][z_window] floats of shared memory; the
-// earlier positions' g are the per-sequence running state), then z and the
-// band combination exactly as score_finalize_kernel forms them (a lane per
-// band, the same shifted two-pass, the same butterfly over the lanes).
-// Every thread of the block calls it; warp 0 writes.
-__device__ __forceinline__ void band_token_scores(const DevState& st, const Dims& dm, int seq, int nc0, int pos,
-                                                  float* win) {
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+// The band kinds' scores of the new token at slot nc0: the per-band z and
+// window means the band CTAs stored, combined exactly as
+// score_finalize_kernel combines them (a lane per band, the same butterfly
+// over the lanes).  One warp calls it.
+__device__ __forceinline__ void band_token_combine(const DevState& st, const Dims& dm, int seq, int nc0, int pos) {
+  const int lane = threadIdx.x & 31;
   const int nb = dm.nA + dm.nB;
-  const int Gm = dm.G - 1;
-  const int w = dm.z_window;
-  const int n = pos >= 1 ? min(w, pos) : 0;
-  for (int idx = tid; idx < nb * n; idx += blockDim.x) {
-    const int bb = idx / n, k = idx - bb * n;
-    win[bb * w + k] = __ldcg(st.g_ring + ((size_t)seq * nb + bb) * dm.G + ((pos - k) & Gm));
-  }
-  __syncthreads();
-  if (warp != 0) return;
   const int lpt = nb <= 16 ? 16 : 32;  // the lanes of one token, as in score_finalize_kernel
   const int bl = lane % lpt;
   const bool live = lane < lpt && pos >= 1 && bl < nb;
   float za = 0.f, zb = 0.f, ma = 0.f, mb = 0.f;
   if (live) {
-    const float* row = win + bl * w;  // row[k] = g at position pos - k
     if (dm.kinds & EPIKV_SCORE_BANDZ) {
-      const float gnew = row[0];
-      float dsum = 0.f;
-      for (int k = 0; k < n; ++k) dsum += row[k] - gnew;
-      const float mean_d = dsum / (float)n;
-      float dev = 0.f;
-      for (int k = 0; k < n; ++k) {
-        const float e = (row[k] - gnew) - mean_d;
-        dev = fmaf(e, e, dev);
-      }
-      const float sigma = sqrtf(dev / (float)n);
-      const float z = -mean_d / (sigma + dm.z_eps);
+      const float z = __ldcg(st.ztok + (size_t)(seq * 2) * nb + bl);
       if (bl < dm.nA) za = z; else zb = z;
     }
     if (dm.kinds & EPIKV_SCORE_HSVAR) {
-      float sum = 0.f;
-      for (int k = 0; k < n; ++k) sum += row[k];
-      const float gbar = sum / (float)n;
+      const float gbar = __ldcg(st.ztok + (size_t)(seq * 2 + 1) * nb + bl);
       if (bl < dm.nA) ma = gbar; else mb = gbar;
     }
   }
@@ -891,10 +901,10 @@ __device__ __forceinline__ void token_commit(const DevState& st, const Dims& dm,
 
 // One new token per sequence with the band kinds only: g and the rolling
 // z-score in one launch.  grid (band layers, batch entries), kGThreads
-// threads: each CTA forms its band row's g (band_token_g); the last CTA of a
-// sequence (atomic ticket after a fence; no CTA waits) forms the scores
-// (band_token_scores) and commits the sequence.  Results equal the
-// two-kernel path bit for bit.
+// threads: each CTA forms its band row's g and that band's z and window mean
+// (band_token_g); the last CTA of a sequence (atomic ticket after a fence; no
+// CTA waits) combines them into the scores (band_token_combine) and commits
+// the sequence.  Results equal the two-kernel path bit for bit.
 template <int VPT>
 __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dims dm, BandRows rows,
                                                                  int64_t row_stride,
@@ -919,7 +929,8 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
     return;
   }
   __shared__ int s_last;
-  band_token_g<VPT>(st, dm, rows, row_stride, band, seq, r0, pos, st.hp_parity[seq]);
+  extern __shared__ float win[];  // [z_window]: this band's window of g
+  band_token_g<VPT>(st, dm, rows, row_stride, band, seq, r0, pos, st.hp_parity[seq], win);
   if (tid == 0) {
     __threadfence();
     s_last = atomicAdd(&st.ticket[seq], 1u) == (unsigned)(nb - 1);
@@ -927,18 +938,18 @@ __global__ void __launch_bounds__(kGThreads) bandz_token_kernel(DevState st, Dim
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  extern __shared__ float win[];  // [nb][z_window]
-  band_token_scores(st, dm, seq, nc0, pos, win);  // warp 0 after a block barrier
+  if (tid < 32) band_token_combine(st, dm, seq, nc0, pos);
   if (tid == 32) token_commit(st, dm, seq, nc0, pos);  // meanwhile: they touch disjoint state
 }
 
 // One new token per sequence with a K/V kind (and any band kinds): the whole
 // score update in one launch.  grid (band layers + L or 2L, batch entries),
-// kGThreads threads: the first CTAs form the band rows' g (band_token_g), the
+// kGThreads threads: the first CTAs form the band rows' g, z and window means
+// (band_token_g), the
 // others the (layer, K|V) streams (lag_stream, the multi-token kernel's own
 // code on a one-token call): a layer's K and V in the two halves of a CTA
 // (`half`, when H*d/8 <= 128), else one stream per CTA; the last CTA of a
-// sequence (ticket) forms every kind's score (band_token_scores,
+// sequence (ticket) forms every kind's score (band_token_combine,
 // kv_token_scores) and commits.  Results equal the three-kernel path bit for
 // bit.
 template <int LH>
@@ -963,11 +974,12 @@ __global__ void __launch_bounds__(kGThreads, EPIKV_TOKEN_MINB) token_kernel(DevS
     return;
   }
   __shared__ int s_last;
+  extern __shared__ float win[];  // [z_window] (band CTAs): the band's window of g
   if ((int)blockIdx.x < nbc) {
     const int par = st.hp_parity[seq];
-    if (vpt == 1) band_token_g<1>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
-    else if (vpt == 2) band_token_g<2>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
-    else band_token_g<4>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par);
+    if (vpt == 1) band_token_g<1>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par, win);
+    else if (vpt == 2) band_token_g<2>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par, win);
+    else band_token_g<4>(st, dm, rows, row_stride, blockIdx.x, seq, r0, pos, par, win);
   } else {
     const int sidx = blockIdx.x - nbc;
     const int layer = half ? sidx : sidx >> 1;
@@ -984,10 +996,9 @@ __global__ void __launch_bounds__(kGThreads, EPIKV_TOKEN_MINB) token_kernel(DevS
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  extern __shared__ float win[];  // [nb][z_window] (band kinds)
-  // three warps at once, on disjoint state: the band scores (warp 0, after a
-  // block barrier), the K/V scores (warp 1) and the commit (warp 2)
-  if (nbc) band_token_scores(st, dm, seq, nc0, pos, win);
+  // three warps at once, on disjoint state: the band scores (warp 0), the
+  // K/V scores (warp 1) and the commit (warp 2)
+  if (nbc && tid < 32) band_token_combine(st, dm, seq, nc0, pos);
   if (tid >= 32 && tid < 64) kv_token_scores(st, dm, seq, nc0, pos);
   if (tid == 64) token_commit(st, dm, seq, nc0, pos);
 }
@@ -1037,7 +1048,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
   const int vpt = vr <= kGThreads ? 1 : vr <= 2 * kGThreads ? 2 : 4;  // band row vectors per thread
   if (max_new == 1 && !(dm.kinds & kKvKinds)) {  // a decode step of the band kinds: one fused launch
     const dim3 grid(nb, n_seq);
-    const size_t wsm = (size_t)nb * dm.z_window * sizeof(float);  // the last CTA's staged windows
+    const size_t wsm = (size_t)dm.z_window * sizeof(float);  // a band CTA's window of g
     auto go = [&](auto kern) { pdl_launch(kern, grid, kGThreads, wsm, stream, st, dm, rows, rs, seq_ids, cu_new); };
     if (vpt == 1) go(bandz_token_kernel<1>);
     else if (vpt == 2) go(bandz_token_kernel<2>);
@@ -1048,7 +1059,7 @@ cudaError_t launch_score_update(const DevState& st, const Dims& dm, int n_seq, c
   if (max_new == 1 && dm.L <= 64) {  // a decode step with a K/V kind: one fused launch
     const int half = dm.H * dm.d / 8 <= 128;  // a layer's K and V streams share a CTA
     const dim3 grid((band ? nb : 0) + (half ? dm.L : 2 * dm.L), n_seq);
-    const size_t wsm = band ? (size_t)nb * dm.z_window * sizeof(float) : 0;
+    const size_t wsm = band ? (size_t)dm.z_window * sizeof(float) : 0;
     auto go = [&](auto kern) {
       pdl_launch(kern, grid, kGThreads, wsm, stream, st, dm, rows, rs, *kv, seq_ids, cu_new, vpt, half);
     };
