@@ -194,12 +194,13 @@ struct RadixShared {
 };
 
 // The M-th largest key_at(i) over i in [c0, c1), 0 < M <= c1 - c0, by a
-// 4-pass 8-bit radix select: *theta is that key and *need_eq the number of
-// keys equal to it that belong to the M largest (the lowest slots first).
+// 4-pass 8-bit radix select: *theta is that key, *need_eq the number of
+// keys equal to it that belong to the M largest (the lowest slots first) and
+// *total_eq (when given) the number of keys equal to it.
 // Every thread of the block (NT threads) calls it.
 template <int NT = kSelThreads, typename KeyAt>
 __device__ __forceinline__ void radix_select(const KeyAt& key_at, int c0, int c1, int M, RadixShared& rs,
-                                             uint32_t* theta, int* need_eq) {
+                                             uint32_t* theta, int* need_eq, int* total_eq = nullptr) {
   const int tid = threadIdx.x;
   __syncthreads();  // every thread has read the previous call's result
   if (tid == 0) {
@@ -249,6 +250,7 @@ __device__ __forceinline__ void radix_select(const KeyAt& key_at, int c0, int c1
   }
   *theta = rs.prefix;
   *need_eq = (int)rs.remaining;
+  if (total_eq) *total_eq = (int)rs.hist[rs.prefix & 255u];  // the last pass's bin: keys equal to theta
 }
 
 template <bool kChunked>
@@ -334,40 +336,51 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
 
   // ---- radix select of the M-th largest key among the candidates
   uint32_t theta = 0xFFFFFFFFu;
-  int need_eq = 0;
-  if (M > 0) radix_select(key_at, c0, c1, M, rs, &theta, &need_eq);
+  int need_eq = 0, total_eq = 0;  // no key is 0xFFFFFFFF (order_key), so M == 0 keeps no candidate
+  if (M > 0) radix_select(key_at, c0, c1, M, rs, &theta, &need_eq, &total_eq);
 
   // ---- ordered scans over contiguous per-thread slot ranges
   const int per = (n + kSelThreads - 1) / kSelThreads;
   const int a = min(n, tid * per), e = min(n, a + per);
-  int eq_local = 0;
-  for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (key_at(i) == theta);
-  int tot;
-  const int eq_base = block_exclusive_scan(eq_local, &tot, sh_scan);
+  // when every key equal to theta is kept (the usual case), which of them
+  // come first does not matter and the count before each thread is not needed
+  const bool all_eq = need_eq == total_eq;
+  int eq_base = 0;
+  if (!all_eq) {  // uniform across the block
+    int eq_local = 0;
+    for (int i = max(a, c0); i < min(e, c1); ++i) eq_local += (key_at(i) == theta);
+    int tot;
+    eq_base = block_exclusive_scan(eq_local, &tot, sh_scan);
+  }
 
+  auto kept_slot = [&](int i, int& eqs) -> bool {
+    if (i < c0 || i >= c1) return true;
+    const uint32_t k = key_at(i);
+    return k > theta || (k == theta && (all_eq || eqs++ < need_eq));
+  };
   int keep_local = 0, first_ev = INT_MAX;
+  uint64_t kmask = 0;  // with at most 64 slots per thread: bit i - a set when slot i is kept
   {
     int eqs = eq_base;
     for (int i = a; i < e; ++i) {
-      bool keep = (i < c0) || (i >= c1);
-      if (!keep) {
-        const uint32_t k = key_at(i);
-        keep = k > theta || (k == theta && eqs++ < need_eq);
+      if (kept_slot(i, eqs)) {
+        ++keep_local;
+        if (per <= 64) kmask |= 1ull << (i - a);
+      } else {
+        first_ev = min(first_ev, i);
       }
-      if (keep) ++keep_local; else first_ev = min(first_ev, i);
     }
   }
   int n_kept;
   const int keep_base = block_exclusive_scan(keep_local, &n_kept, sh_scan);
   {
-    int eqs = eq_base, o = keep_base;
-    for (int i = a; i < e; ++i) {
-      bool keep = (i < c0) || (i >= c1);
-      if (!keep) {
-        const uint32_t k = key_at(i);
-        keep = k > theta || (k == theta && eqs++ < need_eq);
-      }
-      if (keep) out[o++] = i;
+    int o = keep_base;
+    if (per <= 64) {  // uniform across the block
+      for (uint64_t m = kmask; m; m &= m - 1) out[o++] = a + __ffsll((long long)m) - 1;
+    } else {
+      int eqs = eq_base;
+      for (int i = a; i < e; ++i)
+        if (kept_slot(i, eqs)) out[o++] = i;
     }
   }
   const int fe = min(block_min(first_ev, sh_scan), n_kept);
