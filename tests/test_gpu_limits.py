@@ -60,6 +60,30 @@ def test_largest_windows_and_band_count(gpu_lib):
     sess.close()
 
 
+@pytest.mark.parametrize("kinds", [BANDZ | HSVAR, BANDZ | HSVAR | LAGKV], ids=["band-kinds", "with-lagkv"])
+def test_largest_windows_and_band_count_one_token_calls(gpu_lib, kinds):
+    """The decode-step kernels at the limits: 32 band layers (the last CTA
+    combines 32 per-band z values and window means over all 32 lanes) and
+    windows of 1,024, one token per call past position 1,100, every score
+    compared with the fp64 oracle (bandz_token_kernel for the band kinds
+    alone, token_kernel with Lag-KV)."""
+    model = gen.TraceModel(0xE91C0204, num_layers=32, hidden=64, num_kv_heads=1, head_dim=8,
+                           band_a=tuple(range(16)), band_b=tuple(range(16, 32)))
+    T = 1180
+    sess = Session(model, n_seq=1, kinds=kinds, layout=E.EPIKV_LAYOUT_PAGED, max_tokens=T, max_new=400,
+                   prefill=(3,), policies=(BANDZ,), z_window=1024, lag_window=1024)
+    ref = OracleTrace(model, sess.dt.tabs, 0, T, kinds, z_window=1024, lag_window=1024)
+    while sess.n_seen[0] < 1100:
+        sess.score_update([(0, min(400, 1100 - sess.n_seen[0]))])
+    while sess.n_seen[0] < T:
+        sess.score_update([(0, 1)])
+    for kind in (k for k in (BANDZ, HSVAR, LAGKV) if kinds & k):
+        p_, s_ = sess.read(0, kind)
+        ref.check(kind, p_, s_, f"32 bands, windows 1024, one-token calls, kind {kind}")
+    assert sess.error() == (E.EPIKV_OK, 0)
+    sess.close()
+
+
 def test_three_hundred_sequences_in_one_call(gpu_lib):
     model = gen.TraceModel(0xE91C0203, num_layers=2, hidden=64, num_kv_heads=1, head_dim=16,
                            band_a=(0,), band_b=(1,))
