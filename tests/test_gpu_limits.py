@@ -107,3 +107,37 @@ def test_three_hundred_sequences_in_one_call(gpu_lib):
         check_compaction(sess, b, sess.read(b, policies[b])[0])
     assert sess.error() == (E.EPIKV_OK, 0)
     sess.close()
+
+
+@pytest.mark.parametrize("hidden,bands", [(8192, 32), (4096, 32), (4096, 15), (2048, 17)],
+                         ids=["D8192_32bands", "D4096_32bands", "D4096_15bands", "D2048_17bands"])
+def test_band_decode_kernel_widths_and_band_counts(gpu_lib, hidden, bands):
+    """The band-only decode kernel at the hidden widths that change its
+    per-thread vectors (one, two or four 16-byte vectors of each row) with up
+    to 32 band layers (the last CTA of a sequence combines 32 z values).
+    One-token calls are compared with the fp64 oracle and, bit for bit, with
+    the same trace scored in 40-token calls."""
+    nA = bands // 2
+    model = gen.TraceModel(0xE91C0205 + hidden + bands, num_layers=bands, hidden=hidden, num_kv_heads=1,
+                           head_dim=8, band_a=tuple(range(nA)), band_b=tuple(range(nA, bands)))
+    T = 120
+    kinds = BANDZ | HSVAR
+    out = []
+    for chunk in (1, 40):
+        sess = Session(model, n_seq=2, kinds=kinds, layout=E.EPIKV_LAYOUT_CONTIGUOUS, max_tokens=T, max_new=chunk,
+                       prefill=(0, 0), policies=(BANDZ, HSVAR))
+        while sess.n_seen[0] < T:
+            n = min(chunk, T - sess.n_seen[0])
+            sess.score_update([(0, n), (1, n)])
+        out.append([[sess.read(b, k)[1] for k in (BANDZ, HSVAR)] for b in range(2)])
+        if chunk == 1:
+            for b in range(2):
+                ref = OracleTrace(model, sess.dt.tabs, b, T, kinds)
+                for k in (BANDZ, HSVAR):
+                    pos, sc = sess.read(b, k)
+                    ref.check(k, pos, sc, f"D={hidden}, {bands} bands, seq {b}, kind {k}")
+        assert sess.error() == (E.EPIKV_OK, 0)
+        sess.close()
+    for b in range(2):
+        for one, many in zip(out[0][b], out[1][b]):
+            np.testing.assert_array_equal(one, many)
