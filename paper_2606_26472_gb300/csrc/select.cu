@@ -10,7 +10,10 @@
 // (scores of every kind and positions) is then compacted in place, which is
 // safe in increasing order because kept[i] >= i.  When the cache has at most
 // kSelStagedMax slots the candidates' keys are first staged in shared memory,
-// and the radix passes and scans read them there.
+// and the radix passes and scans read them there; when the metadata columns
+// (at most kFusedCols) and the kept list fit beside them, the columns are
+// staged in the same loads, so the moved rows are written from shared memory
+// (coalesced) as soon as the kept list is known.
 //
 // Chunk-level selection (select_chunk = C > 1; the paper names chunk-level
 // scoring as future work, Sec. 5): a first pass gives every candidate slot the
@@ -188,6 +191,13 @@ __device__ __forceinline__ void compact_metadata(const DevState& st, const Dims&
   }
 }
 
+// Metadata columns (score kinds + positions) the selection stages beside its
+// keys; contexts with more score kinds move their metadata after selecting.
+constexpr int kFusedCols = 3;
+#ifndef EPIKV_SEL_FUSED_META
+#define EPIKV_SEL_FUSED_META 1  // 0: the metadata always moved after selecting (compact_metadata)
+#endif
+
 struct RadixShared {
   uint32_t hist[256];
   uint32_t prefix, mask, remaining;
@@ -322,8 +332,53 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   // for the cache (every later pass reads them there instead of from L2)
   extern __shared__ uint32_t skey[];
   const bool staged = staged_cap >= c1 - c0;
+  // With at most kFusedCols metadata columns (each kind's scores, then the
+  // positions) and room for all of them, the cache's columns are staged too,
+  // from the first candidate on (no slot before it moves): the kept rows are
+  // then written from shared memory as the kept list is emitted, with no
+  // round trip after the selection.
+  __shared__ uint32_t* s_col[kNumKinds + 1];
+  __shared__ int s_ncol;
+  if (tid == 0) {
+    int q = 0;
+    for (int k = 0; k < kNumKinds; ++k)
+      if (st.score[k]) s_col[q++] = reinterpret_cast<uint32_t*>(st.score[k]) + (size_t)seq * dm.T;
+    s_col[q++] = reinterpret_cast<uint32_t*>(st.pos) + (size_t)seq * dm.T;
+    s_ncol = q;
+  }
+  __syncthreads();
+  const int ncol = s_ncol;
+  const int kpad = (c1 - c0 + 3) & ~3;
+  const bool fused = EPIKV_SEL_FUSED_META && staged && ncol <= kFusedCols &&
+                     (int64_t)kpad + (int64_t)(ncol + 1) * n <= smem_words;
+  uint32_t* smeta = skey + kpad;  // fused: [ncol][n], column c of slot i at c * n + i
+  int* skept = reinterpret_cast<int*>(smeta + (size_t)ncol * n);  // fused: the kept list
+  uint32_t* col[kFusedCols];
+#pragma unroll
+  for (int c = 0; c < kFusedCols; ++c) col[c] = c < ncol ? s_col[c] : nullptr;
   if (staged) {
-    for (int i = c0 + tid; i < c1; i += kSelThreads) skey[i - c0] = kChunked ? ck[i] : order_key(sc[i]);
+    // U slots per thread with every load in flight before the stores
+    constexpr int U = 4;
+    const int hi = fused ? n : c1;
+    for (int i0 = c0 + tid; i0 < hi; i0 += U * kSelThreads) {
+      uint32_t kv[U], mv[U][kFusedCols];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int i = i0 + u * kSelThreads;
+        if (i < c1) kv[u] = kChunked ? ck[i] : order_key(sc[i]);
+#pragma unroll
+        for (int c = 0; c < kFusedCols; ++c)
+          if (fused && c < ncol && i < n) mv[u][c] = __ldcg(col[c] + i);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int i = i0 + u * kSelThreads;
+        if (i < c1) skey[i - c0] = kv[u];
+#pragma unroll
+        for (int c = 0; c < kFusedCols; ++c)
+          if (fused && c < ncol && i < n) smeta[c * n + i] = mv[u][c];
+      }
+    }
     __syncthreads();
   }
   auto key_at = [&](int i) -> uint32_t {
@@ -376,7 +431,12 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
   {
     int o = keep_base;
     if (per <= 64) {  // uniform across the block
-      for (uint64_t m = kmask; m; m &= m - 1) out[o++] = a + __ffsll((long long)m) - 1;
+      for (uint64_t m = kmask; m; m &= m - 1) {
+        const int i = a + __ffsll((long long)m) - 1;
+        out[o] = i;
+        if (fused) skept[o] = i;
+        ++o;
+      }
     } else {
       int eqs = eq_base;
       for (int i = a; i < e; ++i)
@@ -388,7 +448,17 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(DevState st, Dims d
 
   // ---- compact slot metadata in place (kept[i] >= i, increasing i); the
   // staged keys are no longer needed, so their shared memory stages it
-  compact_metadata(st, dm, seq, out, fe, n_kept, skey, smem_words);
+  // (fused: every row from the staged columns, coalesced stores)
+  if (fused) {
+    for (int o = fe + tid; o < n_kept; o += kSelThreads) {
+      const int i = skept[o];
+#pragma unroll
+      for (int c = 0; c < kFusedCols; ++c)
+        if (c < ncol) col[c][o] = smeta[c * n + i];
+    }
+  } else {
+    compact_metadata(st, dm, seq, out, fe, n_kept, skey, smem_words);
+  }
   if (tid == 0) {
     st.n_cache[seq] = n_kept;
     st.first_changed[seq] = fe;
@@ -903,8 +973,11 @@ __global__ void __launch_bounds__(kSelThreads) layer_union_kernel(DevState st, D
 constexpr int kSelStagedMax = 48 * 1024;  // 192 KiB of u32 words
 static int sel_staged_cap(const Dims& dm) { return dm.T <= kSelStagedMax ? dm.T : 0; }
 static int sel_smem_words(const Dims& dm) {
-  const int64_t meta = (int64_t)(__builtin_popcount((unsigned)dm.kinds) + 1) * dm.T;
-  const int64_t w = meta > sel_staged_cap(dm) ? meta : sel_staged_cap(dm);
+  const int64_t ncol = __builtin_popcount((unsigned)dm.kinds) + 1;  // metadata columns
+  const int64_t meta = ncol * dm.T;
+  int64_t w = meta > sel_staged_cap(dm) ? meta : sel_staged_cap(dm);
+  const int64_t fused = ((int64_t)dm.T + 3) / 4 * 4 + (ncol + 1) * dm.T;  // keys, every column, the kept list
+  if (ncol <= kFusedCols && fused <= kSelStagedMax && fused > w) w = fused;
   return (int)(w < kSelStagedMax ? w : kSelStagedMax);
 }
 static size_t sel_smem(const Dims& dm) { return (size_t)sel_smem_words(dm) * sizeof(uint32_t); }
