@@ -97,17 +97,22 @@ __host__ __device__ inline int pre_entries(int cap) { return (cap + 32) / 32 * 3
 // The batch entries that evicted, in batch order, into list; with pre, the
 // prefix sums of their moved rows per stream (pre[k] = rows of entries
 // before the k-th).  One warp; every CTA of both kernels builds the same.
+// Every entry's moved rows are loaded first (list holds them, list_ints(n_seq)
+// >= n_seq words), all loads in flight together, then scanned in place.
 __device__ int evicting_entries(const DevState& st, const Dims& dm, const int32_t* __restrict__ seq_ids,
                                 int n_seq, int* list, int64_t* pre, int lane) {
+#pragma unroll 4
+  for (int b = lane; b < n_seq; b += 32) {
+    const int seq = seq_ids[b];
+    list[b] = (seq >= 0 && seq < dm.S) ? st.n_cache[seq] - st.first_changed[seq] : 0;
+  }
+  __syncwarp();
   int n_ev = 0;
   int64_t acc = 0;
   for (int base = 0; base < n_seq; base += 32) {
     const int b = base + lane;
-    int len = 0;
-    if (b < n_seq) {
-      const int seq = seq_ids[b];
-      if (seq >= 0 && seq < dm.S) len = st.n_cache[seq] - st.first_changed[seq];
-    }
+    const int len = b < n_seq ? list[b] : 0;
+    __syncwarp();  // the chunk's lengths are read before any of its entries is written
     const bool ev = len > 0;
     const unsigned m = __ballot_sync(0xffffffffu, ev);
     int incl = ev ? len : 0;
@@ -118,11 +123,12 @@ __device__ int evicting_entries(const DevState& st, const Dims& dm, const int32_
     }
     if (ev) {
       const int k = n_ev + __popc(m & ((1u << lane) - 1u));
-      list[k] = b;
+      list[k] = b;   // k <= b: an entry already read
       if (pre) pre[k + 1] = acc + incl;
     }
     acc += __shfl_sync(0xffffffffu, incl, 31);
     n_ev += __popc(m);
+    __syncwarp();
   }
   if (pre && lane == 0) pre[0] = 0;
   __syncwarp();
