@@ -318,6 +318,9 @@ __device__ __forceinline__ void transpose_sum(float (&v)[NV], int lane) {
 // KINDS: 0 = whichever K/V kinds the context computes (runtime flags); 1 =
 // the normalised kinds only; 2 = the raw kinds only; 3 = both (compile-time,
 // so a kernel instance holds only the registers its kinds need).
+#ifndef EPIKV_TOKEN_OWN_OFFSET
+#define EPIKV_TOKEN_OWN_OFFSET 1  // 0: one-token calls also look the row up through shared memory
+#endif
 template <int LH, int SEG = kLagSeg, bool HALF = false, int KINDS = 0>
 __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, const KvDev& kv, int seq,
                                            int n_new, int layer, int kvk, int nc0) {
@@ -366,9 +369,16 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
 
   for (int g0 = 0; g0 < n_new; g0 += kLagOffs) {
     const int gn = min(kLagOffs, n_new - g0);
-    __syncthreads();
-    for (int t = tid; t < gn; t += nthr) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
-    __syncthreads();
+    // one-token calls: every thread looks its row up itself (one broadcast
+    // load per warp), so no shared table and none of its two barriers
+    int64_t off1 = 0;
+    if constexpr (SEG == 1 && EPIKV_TOKEN_OWN_OFFSET) {
+      off1 = kv_row_offset(kv, layer, seq, nc0 + g0, dm.T);
+    } else {
+      __syncthreads();
+      for (int t = tid; t < gn; t += nthr) soff[t] = kv_row_offset(kv, layer, seq, nc0 + g0 + t, dm.T);
+      __syncthreads();
+    }
     // rows are prefetched into L2 kLagPf segments ahead of their loads (whole
     // rows of H*d channels, one bulk prefetch each); the group's first ones here
     const uint32_t row_bytes = (uint32_t)hd * 2u;
@@ -389,7 +399,8 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
         bool all_ok = active;
 #pragma unroll
         for (int j = 0; j < SEG; ++j) {
-          offs[j] = (FULL || j < seg) ? soff[i + j] : 0;
+          if constexpr (SEG == 1 && EPIKV_TOKEN_OWN_OFFSET) offs[j] = off1;
+          else offs[j] = (FULL || j < seg) ? soff[i + j] : 0;
           all_ok &= offs[j] >= 0;
         }
         if (FULL && all_ok) {  // every row of the segment mapped: plain loads
