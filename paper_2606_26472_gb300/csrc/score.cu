@@ -370,7 +370,10 @@ __device__ __forceinline__ void lag_stream(const DevState& st, const Dims& dm, c
   for (int g0 = 0; g0 < n_new; g0 += kLagOffs) {
     const int gn = min(kLagOffs, n_new - g0);
     // one-token calls: every thread looks its row up itself (one broadcast
-    // load per warp), so no shared table and none of its two barriers
+    // load per warp), so no shared table and none of its two barriers.  The
+    // SEG == 1 instances run only in the decode-step kernel, whose calls
+    // carry one token per sequence (it rejects n_new > 1), so the group holds
+    // that one row.
     int64_t off1 = 0;
     if constexpr (SEG == 1 && EPIKV_TOKEN_OWN_OFFSET) {
       off1 = kv_row_offset(kv, layer, seq, nc0 + g0, dm.T);
